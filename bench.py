@@ -1,0 +1,390 @@
+#!/usr/bin/env python
+"""Throughput of the PGC hot path on GB300: one JSON line on stdout.
+
+A "step" is one ``pgc_step`` call: every scheduled per-partition gradient,
+the gradient-store commit, and the decode fused with the SGD update, over the
+workload's resident partitions.  ``value`` is steady-state steps/s measured
+with CUDA events on the library's stream (inputs resident in HBM), max over
+ranks.  ``e2e`` is the same metric through the Python API with host buffers:
+the straggler mask goes host->device and the decoded gradient and the new
+parameters come back device->host every step.
+
+  python bench.py [--workload NAME] [--steps K] [--warmup W] [--gpus N]
+  python bench.py --impl reference ...   # the fp64 CPU oracle, same workload
+
+With --gpus N > 1 (under torchrun) each rank runs an independent replica of
+the whole simulated cluster (the path keeps all n workers on one GPU), so the
+scaling is weak and ``value`` is the sum over ranks.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_20739_gb300 import workloads as W  # noqa: E402
+
+METRIC = "PGC steps/s & samples/s at 1 GB300; % of HBM (or bf16 TC) roofline"
+DEFAULT_WORKLOAD = "cr_n8_logistic_d1024"
+L2_BYTES = 129 * 2 ** 20
+KERNEL_NAMES = ["gradient", "commit", "decode"]
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=W.WORKLOAD_ORDER)
+    ap.add_argument("--seed", type=int, default=1)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle sample")
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work (per steady step)
+# ---------------------------------------------------------------------------
+
+def evaluated_rows(w: W.Workload) -> int:
+    """Distinct rows evaluated per steady step: FR computes one partition per
+    group (n/c partitions), CR all n."""
+    rows = w.rows()
+    if w.scheme == "FR":
+        return sum(rows[g * w.c] for g in range(w.n // w.c))
+    return sum(rows)
+
+
+def grad_bytes_per_row(w: W.Workload) -> int:
+    esz = 2 if w.dtype == "bf16" else 4
+    return w.d * esz + 4
+
+
+def roofline_model(w: W.Workload, peaks: dict):
+    """(bound, algorithmic units per gradient launch, unit name, peak)."""
+    rows = evaluated_rows(w)
+    if w.loss == "softmax" and w.K >= 256:
+        flops = 2.0 * 2.0 * rows * w.d * w.K
+        return "tensor", flops, "TFLOP/s", peaks.get("bf16_tflops_sustained") or 1700.0
+    return "hbm", float(rows * grad_bytes_per_row(w)), "GB/s", peaks.get("hbm_gbs") or 6800.0
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_20739_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, f), "rb") as fh:
+                h.update(f.encode())
+                h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary, if the kernel sources have not changed since it was taken."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    e = d.get(workload)
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ---------------------------------------------------------------------------
+# the fp64 oracle on the host cores (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------
+
+def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 2):
+    """Steady steps/s of the oracle as it stands: warm-up step 0 untimed, then
+    steady steps until the budget is spent."""
+    from oracle import pgc_oracle as O
+    S = {"FR": O.FR, "CR": O.CR}
+    L = {"logistic": O.LOGISTIC, "lsq": O.LSQ, "softmax": O.SOFTMAX}
+    Xf = [W.features_as_float(X, w.dtype) for X in Xs]
+    o = O.PGCOracle(S[w.scheme], w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
+    o.step(masks[0])
+    t0 = time.perf_counter()
+    k = 0
+    while True:
+        o.step(masks[(1 + k) % len(masks)])
+        k += 1
+        el = time.perf_counter() - t0
+        if (el >= budget_s and k >= min_steps) or el >= 4 * budget_s:
+            break
+    return k / el, k, el
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (independent replicas; only timing is reduced)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# arms
+# ---------------------------------------------------------------------------
+
+def default_steps(w: W.Workload) -> int:
+    per_step_bytes = evaluated_rows(w) * grad_bytes_per_row(w)
+    est_s = max(per_step_bytes / 5.0e12, 20e-6)
+    return int(min(20000, max(20, 2.0 / est_s)))
+
+
+def run_ours(args):
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2607_20739_gb300 import binding as B
+
+    w = W.WORKLOADS[args.workload]
+    K_steps = args.steps or default_steps(w)
+    Wu = max(3, args.warmup)
+    Xs, ys = W.make_partitions(w, args.seed)
+    masks = W.make_masks(w, K_steps + Wu + 1, args.seed + 1000)
+
+    stream = torch.cuda.Stream(device=dev)
+    g = B.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream)
+    g.load(Xs, ys)
+    P = w.K * w.d
+    gout = torch.empty(P, device=dev)
+    wout = torch.empty(P, device=dev)
+    step_bytes = evaluated_rows(w) * grad_bytes_per_row(w)
+    flush = step_bytes <= L2_BYTES
+    flush_buf = torch.empty(256 * 2 ** 20 // 4, device=dev) if flush else None
+    mptr = [np.ascontiguousarray(masks[t]) for t in range(len(masks))]
+
+    def do_step(t):
+        if flush:
+            with torch.cuda.stream(stream):
+                flush_buf.zero_()
+        g.step(mptr[t], gout, wout, info=False)
+
+    for t in range(Wu):
+        do_step(t)
+    g.sync()
+
+    # ---- device-timed region -------------------------------------------
+    clk = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clk.start()
+    time.sleep(0.25)
+    g.timing(True)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for t in range(Wu, Wu + K_steps):
+        do_step(t)
+    ev1.record(stream)
+    g.sync()
+    torch.cuda.synchronize(dev)
+    region_ms = ev0.elapsed_time(ev1)
+    tim = g.timing_read()
+    g.timing(False)
+    clocks = clk.stop()
+    barrier(world)
+    step_ms_sum = sum(tim["ms"])
+    ms_per_step = (step_ms_sum if flush else region_ms) / K_steps
+    ms_per_step = max_over_ranks(ms_per_step, world, dev)
+    value = world * 1000.0 / ms_per_step
+
+    # ---- roofline of the dominant kernel (gradient group) ----------------
+    peaks, peak_src = load_peaks()
+    bound, units, unit, peak = roofline_model(w, peaks)
+    grad_ms = tim["ms"][0] / max(1, tim["steps"])
+    if unit == "GB/s":
+        achieved = units / (grad_ms * 1e-3) / 1e9
+    else:
+        achieved = units / (grad_ms * 1e-3) / 1e12
+    traffic = recorded_traffic(w.name)
+
+    # ---- end to end through the public API with host buffers -------------
+    g2 = g
+    gh = torch.empty(P, dtype=torch.float32).pin_memory()
+    wh = torch.empty(P, dtype=torch.float32).pin_memory()
+    e2e_steps = max(10, min(K_steps, 2000))
+    barrier(world)
+    t0 = time.perf_counter()
+    for t in range(e2e_steps):
+        g2.step(mptr[t % len(mptr)], gh, wh, info=False)
+    e2e_s = time.perf_counter() - t0
+    e2e_s = max_over_ranks(e2e_s, world, dev)
+    e2e_value = world * e2e_steps / e2e_s
+
+    # ---- cpu baseline (rank 0, N = 1 only) -------------------------------
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, k, el = time_oracle(w, Xs, ys, masks, args.cpu_seconds)
+        cpu = {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"{k} steady steps of the full {w.name} workload after the warm-up step "
+                         f"({el:.1f} s, fp64 numpy, BLAS threads = all cores)"}
+    g.close()
+
+    uniq = evaluated_rows(w)
+    line = {
+        "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K_steps, "warmup": Wu,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32" if w.dtype == "f32" else "bf16-in/f32-acc",
+        "data": f"synthetic, seeded (seed {args.seed}); {w.features} features, planted-model labels, "
+                f"{w.delays} straggler delays",
+        "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
+                   "rows_per_partition": w.m, "features": w.dtype, "parallelism": f"replicas{world}",
+                   "l2": ("flushed between steps (256 MiB write, excluded from step time)" if flush else
+                          f"inputs larger than L2: {step_bytes / 2**20:.0f} MiB streamed per step")},
+        "samples_per_s_unique": value * uniq,
+        "samples_per_s_worker": value * sum(w.rows()),
+        "kernel_ms_per_step": {KERNEL_NAMES[i]: tim["ms"][i] / max(1, tim["steps"]) for i in range(3)},
+        "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                     "peak_source": peak_src, "kernel": "gradient (K1 streaming row kernel)" if w.loss != "softmax"
+                     else "gradient (softmax)", "traffic": traffic,
+                     "algorithmic_per_launch": units},
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": w.n,
+                "d2h_bytes_per_step": 2 * P * 4},
+        "gpu_launches": int(sum(tim["launches"])),
+        "clocks": clocks,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    w = W.WORKLOADS[args.workload]
+    K_steps = args.steps or 3
+    Xs, ys = W.make_partitions(w, args.seed)
+    masks = W.make_masks(w, K_steps + max(3, args.warmup) + 1, args.seed + 1000)
+    budget = min(args.cpu_seconds, 60.0)
+    v, k, el = time_oracle(w, Xs, ys, masks, budget, min_steps=min(K_steps, 3))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "steps/s", "n_gpus": world, "steps": k,
+        "warmup": 1, "ms_per_step": 1000.0 / v, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": f"synthetic, seeded (seed {args.seed})",
+        "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
+                   "rows_per_partition": w.m},
+        "cpu_baseline": {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": f"{k} steady steps after the warm-up step ({el:.1f} s)"},
+        "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

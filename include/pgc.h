@@ -1,0 +1,213 @@
+/*
+ * pgc.h — C ABI of libpgc, the GB300 (sm_103a) hot path of Pipelined
+ * Gradient Coding (PGC).
+ *
+ * One GPU simulates an n-worker PGC training step that tolerates s
+ * stragglers (c = s + 1 partitions per worker).  Every call is ordered on the
+ * CUDA stream given to pgc_create.  A context is not thread-safe.
+ *
+ * Status codes: every int-returning call returns PGC_OK (0) or a negative
+ * PGC_E* code; pgc_strerror turns a code into text.  On any error the
+ * context's state (step counter, parameters, stores) is unchanged, except for
+ * PGC_ECUDA / PGC_ETIMEOUT which leave the context unusable (destroy it).
+ *
+ * Layouts: features of partition D_k are row-major [m_k][d] (fp32 or bf16
+ * bits); labels are float32 [m_k] (logistic: 0/1, least squares: real) or
+ * int32 [m_k] class indices (softmax).  Parameters beta are float32 [K][d]
+ * row-major (K = 1 for logistic and least squares).
+ */
+#ifndef PGC_H_
+#define PGC_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define PGC_OK        0
+#define PGC_EINVAL   (-1)  /* bad argument (sizes, enum, NULL pointer)       */
+#define PGC_EMASK    (-2)  /* straggler mask is not exactly s ones, n-s zeros */
+#define PGC_ESTATE   (-3)  /* call out of order (e.g. step before load)      */
+#define PGC_ENOMEM   (-4)  /* device or pinned-host allocation failed        */
+#define PGC_ECUDA    (-5)  /* a CUDA runtime call or kernel failed           */
+#define PGC_ENOTSUP  (-6)  /* valid but unsupported combination             */
+#define PGC_ETIMEOUT (-7)  /* a bounded device-side wait gave up            */
+
+/* ---- enumerations (passed as int32) ------------------------------------ */
+/* Dataset placement, §III: FR needs c | n; CR places cyclically.          */
+#define PGC_FR 0
+#define PGC_CR 1
+/* Per-sample loss f: logistic cross-entropy (y in {0,1}), least squares
+ * (1/2)(x.beta - y)^2, softmax cross-entropy over K classes.             */
+#define PGC_LOGISTIC 0
+#define PGC_LSQ      1
+#define PGC_SOFTMAX  2
+/* Storage type of the features.                                           */
+#define PGC_F32  0
+#define PGC_BF16 1
+
+typedef struct pgc_ctx pgc_ctx;
+
+/* Filled by pgc_step.  The arrays are owned by the caller and may be NULL. */
+typedef struct pgc_step_info {
+  int64_t  t;               /* index of the step just taken (0 = warm-up)    */
+  int32_t  slot;            /* o_t = (t - 1) mod c written this step; -1 at t = 0 */
+  int32_t  received;        /* n - s coded gradients decoded                 */
+  int32_t *eval_partition;  /* [n]: partition W_i evaluated; -1 at t = 0     */
+  int32_t *fr_rep;          /* [n/c] (FR only): worker that represents group j */
+} pgc_step_info;
+
+/*
+ * pgc_create — allocate a PGC run (§III problem statement, §IV-A, §V-B).
+ *   out      : receives the context (set to NULL on error).
+ *   n, s     : workers and tolerated stragglers; 1 <= c = s + 1 <= n; FR
+ *              additionally needs c | n.  n <= 1024.
+ *   scheme   : PGC_FR or PGC_CR.   loss: PGC_LOGISTIC, PGC_LSQ, PGC_SOFTMAX.
+ *   dtype    : storage of the features (PGC_F32 or PGC_BF16).
+ *   d        : features per sample (>= 1).  K: classes (1 unless softmax;
+ *              softmax needs 2 <= K <= 4096).
+ *   rows     : host array [n], rows m_k >= 1 of partition D_k.
+ *   lr       : learning rate eta of beta <- beta - eta * ghat (§III).
+ *   w0       : host array [K*d] initial beta, or NULL for zeros.
+ *   stream   : cudaStream_t every call is ordered on (NULL = legacy stream).
+ * Allocates all device state (partitions, parameters, the per-owner gradient
+ * stores, slot totals, scratch).  Errors: PGC_EINVAL, PGC_ENOTSUP,
+ * PGC_ENOMEM, PGC_ECUDA.  Argument checks happen before any CUDA call.
+ */
+int pgc_create(pgc_ctx **out, int32_t n, int32_t s, int32_t scheme, int32_t loss,
+               int32_t dtype, int64_t d, int64_t K, const int64_t *rows, float lr,
+               const float *w0, void *stream);
+
+/*
+ * pgc_load_partitions — copy the n partitions into device memory (§III: the
+ * partitions are placed before training).  X[k] points to [m_k][d] features
+ * of the create-time dtype, y[k] to m_k labels (float32, or int32 for
+ * softmax).  on_device != 0: the pointers are device pointers; otherwise host
+ * pointers.  The library keeps its own copy; the caller may free its buffers
+ * after the call returns.  May be called again to replace the data; it does
+ * not reset the step counter.  Errors: PGC_EINVAL (NULL entry), PGC_ECUDA.
+ */
+int pgc_load_partitions(pgc_ctx *ctx, const void *const *X, const void *const *y,
+                        int32_t on_device);
+
+/*
+ * pgc_step — one PGC training step t (§IV-A PGC-FR, §V-B PGC-CR).
+ *   straggler_mask : host array [n]; 1 marks a straggler, 0 a worker whose
+ *                    coded gradient reaches the master.  Exactly s ones.
+ *   grad_out       : [K*d] float32, receives the decoded gradient ghat^(t)
+ *                    (NULL: not returned).
+ *   w_out          : [K*d] float32, receives beta^(t+1) (NULL: not returned).
+ *   outputs_on_device : != 0: grad_out / w_out are device pointers and the
+ *                    call returns without waiting for the GPU; 0: host
+ *                    pointers, the call waits for the copies.
+ *   info           : may be NULL; receives t, o_t and the schedule indices.
+ * Step 0 is the warm-up: every worker evaluates all c of its partitions at
+ * beta^(0).  From step 1 on, worker W_i evaluates only the partition in its
+ * slot o_t = (t-1) mod c; stragglers still evaluate and store.  FR workers of
+ * one group evaluate the same partition at the same beta, so it is computed
+ * once per group.  The decode uses the coded gradients of the n - s received
+ * workers with the coefficients of §IV-A (FR: one per group, times 1/n) or
+ * §V-B (CR: times 1/((n-s)c)), derived on the device from the mask, and is
+ * fused with the SGD update.  Errors: PGC_ESTATE (no partitions loaded),
+ * PGC_EMASK, PGC_EINVAL, PGC_ECUDA, PGC_ETIMEOUT.
+ */
+int pgc_step(pgc_ctx *ctx, const uint8_t *straggler_mask, float *grad_out, float *w_out,
+             int32_t outputs_on_device, pgc_step_info *info);
+
+/*
+ * pgc_loss — F(beta^(t)) = (1 / sum_k m_k) sum over all samples of f, at the
+ * current parameters (§III).  Untimed helper; waits for the GPU.
+ * Errors: PGC_ESTATE, PGC_EINVAL, PGC_ECUDA.
+ */
+int pgc_loss(pgc_ctx *ctx, double *loss_out);
+
+/*
+ * pgc_sync — wait for every call issued on the context's stream and report
+ * a device-side failure (PGC_ETIMEOUT if a bounded wait gave up, PGC_EMASK
+ * if the decode kernel saw an invalid mask).  Steps with device outputs do
+ * not wait; call this before trusting their results.
+ */
+int pgc_sync(pgc_ctx *ctx);
+
+/* pgc_destroy — free everything; NULL is accepted.  Returns PGC_OK. */
+int pgc_destroy(pgc_ctx *ctx);
+
+/* pgc_strerror — static text for a status code. */
+const char *pgc_strerror(int32_t code);
+
+/* ---- host-only helpers: pure index arithmetic, no CUDA call ------------- */
+
+/*
+ * pgc_placement — the partitions each worker holds (§III; §IV-A for FR,
+ * §V-B for CR), table[i*c + l] = partition in slot l of worker W_i.
+ * table: host [n*c].  Errors: PGC_EINVAL.
+ */
+int pgc_placement(int32_t scheme, int32_t n, int32_t s, int32_t *table);
+
+/*
+ * pgc_schedule — partition each worker evaluates at step t (§IV-A, §V-B):
+ * eval_partition[i] (host [n]) = the partition in slot (t-1) mod c of W_i,
+ * or -1 for every worker at t = 0; *slot = (t-1) mod c or -1.
+ * Errors: PGC_EINVAL.
+ */
+int pgc_schedule(int32_t scheme, int32_t n, int32_t s, int64_t t,
+                 int32_t *eval_partition, int32_t *slot);
+
+/* ---- inspection of device state (tests; each call waits for the GPU) ---- */
+
+/*
+ * pgc_get_store — copy worker W_i's stored gradient in slot l (the gradient
+ * of the partition in slot l of its holdings, as last evaluated) to host
+ * out[K*d].  FR workers of one group share one store.  Errors: PGC_EINVAL,
+ * PGC_ESTATE, PGC_ECUDA.
+ */
+int pgc_get_store(pgc_ctx *ctx, int32_t worker, int32_t slot, float *out);
+
+/*
+ * pgc_get_decode — the decoding coefficients the device derived from the
+ * last step's mask: coeff[i] (host [n]) = weight a_i of W_i's coded gradient
+ * (§IV-A: 1/n for each FR group's representative; §V-B: 1/((n-s)c) for each
+ * received CR worker; 0 otherwise).  Errors: PGC_ESTATE, PGC_ECUDA.
+ */
+int pgc_get_decode(pgc_ctx *ctx, float *coeff);
+
+/* pgc_get_weights — copy the current beta to host out[K*d]. */
+int pgc_get_weights(pgc_ctx *ctx, float *out);
+
+/* pgc_set_weights — overwrite beta with host w[K*d] (teacher forcing in
+ * tests; also the checkpoint-restore path).  Errors: PGC_EINVAL, PGC_ECUDA. */
+int pgc_set_weights(pgc_ctx *ctx, const float *w);
+
+/* pgc_step_count — number of steps taken so far (host-side counter). */
+int64_t pgc_step_count(const pgc_ctx *ctx);
+
+/* ---- measurement ---------------------------------------------------------- */
+
+/* Kernel groups of one step, as counted and timed below. */
+#define PGC_KGRAD   0   /* per-partition gradient kernels                      */
+#define PGC_KCOMMIT 1   /* gradient-store commit                               */
+#define PGC_KDECODE 2   /* decode coefficients + decode + SGD                  */
+#define PGC_NKGROUPS 3
+
+/*
+ * pgc_timing — enable != 0 starts recording CUDA events on the context's
+ * stream around each kernel group of every following step (and clears what
+ * was recorded); 0 stops.  Errors: PGC_EINVAL, PGC_ECUDA.
+ */
+int pgc_timing(pgc_ctx *ctx, int32_t enable);
+
+/*
+ * pgc_timing_read — wait for the stream, then return for each kernel group
+ * the summed device time in milliseconds (ms[PGC_NKGROUPS]) over the steps
+ * recorded since timing was enabled, and the kernels launched by the library
+ * in those steps (launches[PGC_NKGROUPS]).  Either array may be NULL.
+ * *steps_out (nullable) receives the number of recorded steps.
+ */
+int pgc_timing_read(pgc_ctx *ctx, double *ms, int64_t *launches, int64_t *steps_out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PGC_H_ */

@@ -1,0 +1,622 @@
+// Host side of libpgc: argument checks, device state, the step schedule
+// (§IV-A, §V-B), per-phase launch tables and the C ABI of include/pgc.h.
+//
+// Device state of a run (all owned by the context):
+//   X      packed features [sum_k m_k][ld] (rows padded with zeros to ld)
+//   y      packed labels [sum_k m_k] (float32, or int32 classes)
+//   w      beta [K][ld] fp32 (+ a bf16 copy wb for bf16 features)
+//   store  gradient stores [owners][c][K*ld] fp32: owners = n (CR) or n/c
+//          (FR: the c members of a group keep identical stores, §IV-A)
+//   U      slot totals [c][K*ld]: U[o] = sum over owners of store[.][o]
+//   gout   decoded gradient of the last step [K*ld]
+//
+// Phases: phase 0 is the warm-up step t = 0 (every partition evaluated and
+// written to all its holders); phase 1 + o is a steady step with
+// o_t = (t - 1) mod c = o.  Each phase has a fixed list of evaluated
+// partitions, the work items that split their rows across CTAs, and the
+// destination stores of each new gradient.
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/pgc.h"
+#include "pgc_internal.h"
+
+using namespace pgc;
+
+namespace {
+
+constexpr int kItemMaxRows = 8192;
+
+struct Phase {
+  int slot = -1;                        // o, or -1 for the warm-up
+  std::vector<int32_t> parts;           // evaluated partitions (e -> k)
+  std::vector<WorkItem> items;          // row-kernel work items
+  std::vector<int32_t> e_item0;         // CSR of items (or one per e)
+  std::vector<float> e_scale;           // 1 / m_e
+  std::vector<int32_t> e_dest;          // [nE * ndest] store index owner*c+slot
+  int ndest = 1;
+  std::vector<int64_t> e_row0, e_rows, e_zrow0;
+  int64_t z_total = 0, max_rows = 0;
+  int max_item_rows = 1;
+  // device copies
+  WorkItem* d_items = nullptr;
+  int32_t* d_e_item0 = nullptr;
+  float* d_e_scale = nullptr;
+  int32_t* d_e_dest = nullptr;
+  int64_t* d_e_row0 = nullptr;
+  int64_t* d_e_rows = nullptr;
+  int64_t* d_e_zrow0 = nullptr;
+};
+
+bool valid_scheme(int32_t v) { return v == PGC_FR || v == PGC_CR; }
+bool valid_loss(int32_t v) { return v == PGC_LOGISTIC || v == PGC_LSQ || v == PGC_SOFTMAX; }
+bool valid_dtype(int32_t v) { return v == PGC_F32 || v == PGC_BF16; }
+
+int check_nsc(int32_t scheme, int32_t n, int32_t s) {
+  if (!valid_scheme(scheme)) return PGC_EINVAL;
+  if (n < 1 || n > kMaxWorkers || s < 0 || s + 1 > n) return PGC_EINVAL;
+  if (scheme == PGC_FR && n % (s + 1) != 0) return PGC_EINVAL;
+  return PGC_OK;
+}
+
+// Partition in slot l of worker i: FR D_{floor(i/c) c + l} (§IV-A),
+// CR D_{(i + l) mod n} (§V-B).
+inline int32_t held(int32_t scheme, int32_t n, int32_t c, int32_t i, int32_t l) {
+  return scheme == PGC_FR ? (i / c) * c + l : (i + l) % n;
+}
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+}  // namespace
+
+struct pgc_ctx {
+  int32_t n = 0, s = 0, c = 1, scheme = 0, loss = 0, dtype = 0;
+  int64_t d = 0, K = 1, ld = 0, P = 0, Kpad = 0;
+  std::vector<int64_t> rows, row0;
+  int64_t total_rows = 0;
+  float lr = 0.f;
+  cudaStream_t stream = nullptr;
+  int device = 0, sm_count = 148;
+  int variant = -1;          // K1 variant (logistic / least squares)
+  int owners = 0;
+  size_t esize = 4;
+
+  void* X = nullptr;
+  void* y = nullptr;
+  float* w = nullptr;
+  uint16_t* wb = nullptr;
+  float* store = nullptr;
+  float* U = nullptr;
+  float* gout = nullptr;
+  float* partials = nullptr;
+  float* Z = nullptr;
+  float* coeff = nullptr;
+  int* status = nullptr;
+  double* loss_blocks = nullptr;
+  double* loss_out = nullptr;
+  int64_t* loss_desc = nullptr;
+  int64_t loss_chunk = 0;
+  int loss_nblocks = 256;
+  void* tables = nullptr;
+
+  std::vector<Phase> phases;
+  // measurement: events around the kernel groups of each recorded step
+  bool timing = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  int64_t launches[PGC_NKGROUPS] = {0, 0, 0};
+  int64_t timed_steps = 0;
+  bool loaded = false;
+  bool broken = false;
+  bool stepped = false;
+  int64_t t = 0;
+};
+
+namespace {
+
+int cuda_fail(pgc_ctx* ctx, cudaError_t e) {
+  if (e == cudaSuccess) return PGC_OK;
+  if (ctx) ctx->broken = true;
+  return e == cudaErrorMemoryAllocation ? PGC_ENOMEM : PGC_ECUDA;
+}
+
+#define PGC_CK(ctx, expr)                          \
+  do {                                             \
+    cudaError_t _e = (expr);                       \
+    if (_e != cudaSuccess) return cuda_fail(ctx, _e); \
+  } while (0)
+
+// Read and clear nothing: map the device status word to a code.
+int read_status(pgc_ctx* ctx) {
+  int h = 0;
+  cudaError_t e = cudaMemcpyAsync(&h, ctx->status, sizeof(int), cudaMemcpyDeviceToHost, ctx->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
+  if (e != cudaSuccess) return cuda_fail(ctx, e);
+  if (h & kErrWaitTimeout) { ctx->broken = true; return PGC_ETIMEOUT; }
+  if (h & kErrBadMask) { ctx->broken = true; return PGC_EMASK; }
+  if (h) { ctx->broken = true; return PGC_ECUDA; }
+  return PGC_OK;
+}
+
+void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
+  const int n = ctx->n, c = ctx->c;
+  ph.slot = slot;
+  ph.parts.clear();
+  if (slot < 0 || ctx->scheme == PGC_CR) {
+    for (int k = 0; k < n; ++k) ph.parts.push_back(k);
+  } else {
+    for (int g = 0; g < n / c; ++g) ph.parts.push_back(g * c + slot);
+  }
+  const int nE = (int)ph.parts.size();
+  // destinations of each new gradient
+  if (slot < 0 && ctx->scheme == PGC_CR) {
+    ph.ndest = c;
+    for (int e = 0; e < nE; ++e) {
+      const int k = ph.parts[e];
+      for (int l = 0; l < c; ++l) ph.e_dest.push_back(((k - l + n) % n) * c + l);
+    }
+  } else {
+    ph.ndest = 1;
+    for (int e = 0; e < nE; ++e) {
+      const int k = ph.parts[e];
+      if (ctx->scheme == PGC_FR) ph.e_dest.push_back((k / c) * c + (k % c));
+      else ph.e_dest.push_back(((k - slot + n) % n) * c + slot);
+    }
+  }
+  int64_t R = 0;
+  for (int e = 0; e < nE; ++e) {
+    const int k = ph.parts[e];
+    ph.e_scale.push_back(1.0f / (float)ctx->rows[k]);
+    ph.e_row0.push_back(ctx->row0[k]);
+    ph.e_rows.push_back(ctx->rows[k]);
+    ph.e_zrow0.push_back(R);
+    R += ctx->rows[k];
+    ph.max_rows = std::max(ph.max_rows, ctx->rows[k]);
+  }
+  ph.z_total = R;
+  if (ctx->loss != PGC_SOFTMAX) {
+    // split rows into about sm_count * waves items of similar size
+    const double bytes = (double)R * ctx->ld * ctx->esize;
+    const int waves = bytes > 1e9 ? 3 : 1;
+    const int64_t G = (int64_t)ctx->sm_count * waves;
+    const int64_t min_rows = grad_rows_stage_rows(ctx->variant, ctx->ld, ctx->dtype);
+    ph.e_item0.push_back(0);
+    for (int e = 0; e < nE; ++e) {
+      const int64_t m = ph.e_rows[e];
+      int64_t q = (int64_t)std::llround((double)G * (double)m / (double)R);
+      q = std::max<int64_t>(q, 1);
+      q = std::min<int64_t>(q, std::max<int64_t>(1, (m + min_rows - 1) / min_rows));
+      q = std::max<int64_t>(q, (m + kItemMaxRows - 1) / kItemMaxRows);
+      for (int64_t i = 0; i < q; ++i) {
+        const int64_t a = m * i / q, b = m * (i + 1) / q;
+        WorkItem it;
+        it.e = e;
+        it.part = ph.parts[e];
+        it.row0 = ph.e_row0[e] + a;
+        it.rows = b - a;
+        ph.items.push_back(it);
+        ph.max_item_rows = std::max<int>(ph.max_item_rows, (int)(b - a));
+      }
+      ph.e_item0.push_back((int32_t)ph.items.size());
+    }
+  } else {
+    for (int e = 0; e <= nE; ++e) ph.e_item0.push_back(e);
+  }
+}
+
+template <typename T>
+void put(std::vector<uint8_t>& buf, size_t& off, const std::vector<T>& v) {
+  off = align_up(off, 16);
+  const size_t bytes = v.size() * sizeof(T);
+  if (buf.size() < off + bytes) buf.resize(off + bytes);
+  if (bytes) std::memcpy(buf.data() + off, v.data(), bytes);
+  off += bytes;
+}
+
+cudaError_t record_event(pgc_ctx* ctx) {
+  if (!ctx->timing) return cudaSuccess;
+  if (ctx->ev_used == ctx->ev_pool.size()) {
+    cudaEvent_t ev;
+    cudaError_t e = cudaEventCreate(&ev);
+    if (e != cudaSuccess) return e;
+    ctx->ev_pool.push_back(ev);
+  }
+  return cudaEventRecord(ctx->ev_pool[ctx->ev_used++], ctx->stream);
+}
+
+void free_all(pgc_ctx* ctx) {
+  for (cudaEvent_t ev : ctx->ev_pool) cudaEventDestroy(ev);
+  ctx->ev_pool.clear();
+  void* ptrs[] = {ctx->X, ctx->y, ctx->w, ctx->wb, ctx->store, ctx->U, ctx->gout, ctx->partials, ctx->Z,
+                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->loss_desc, ctx->tables};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+}
+
+int copy_out(pgc_ctx* ctx, float* dst, const float* src, int on_device) {
+  // unpad [K][ld] -> [K][d]
+  const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+  PGC_CK(ctx, cudaMemcpy2DAsync(dst, ctx->d * sizeof(float), src, ctx->ld * sizeof(float), ctx->d * sizeof(float),
+                                ctx->K, kind, ctx->stream));
+  return PGC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* pgc_strerror(int32_t code) {
+  switch (code) {
+    case PGC_OK: return "ok";
+    case PGC_EINVAL: return "invalid argument";
+    case PGC_EMASK: return "straggler mask must hold exactly s ones and n-s zeros";
+    case PGC_ESTATE: return "call out of order (partitions not loaded?)";
+    case PGC_ENOMEM: return "out of memory";
+    case PGC_ECUDA: return "CUDA error";
+    case PGC_ENOTSUP: return "unsupported combination";
+    case PGC_ETIMEOUT: return "a bounded device-side wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int pgc_placement(int32_t scheme, int32_t n, int32_t s, int32_t* table) {
+  const int rc = check_nsc(scheme, n, s);
+  if (rc) return rc;
+  if (!table) return PGC_EINVAL;
+  const int c = s + 1;
+  for (int i = 0; i < n; ++i)
+    for (int l = 0; l < c; ++l) table[i * c + l] = held(scheme, n, c, i, l);
+  return PGC_OK;
+}
+
+int pgc_schedule(int32_t scheme, int32_t n, int32_t s, int64_t t, int32_t* eval_partition, int32_t* slot) {
+  const int rc = check_nsc(scheme, n, s);
+  if (rc) return rc;
+  if (t < 0) return PGC_EINVAL;
+  const int c = s + 1;
+  const int o = t == 0 ? -1 : (int)((t - 1) % c);
+  if (slot) *slot = o;
+  if (eval_partition)
+    for (int i = 0; i < n; ++i) eval_partition[i] = o < 0 ? -1 : held(scheme, n, c, i, o);
+  return PGC_OK;
+}
+
+int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss, int32_t dtype, int64_t d,
+               int64_t K, const int64_t* rows, float lr, const float* w0, void* stream) {
+  if (!out) return PGC_EINVAL;
+  *out = nullptr;
+  int rc = check_nsc(scheme, n, s);
+  if (rc) return rc;
+  if (!valid_loss(loss) || !valid_dtype(dtype) || d < 1 || !rows || !std::isfinite(lr)) return PGC_EINVAL;
+  if (loss == PGC_SOFTMAX ? (K < 2 || K > 4096) : K != 1) return PGC_EINVAL;
+  for (int k = 0; k < n; ++k)
+    if (rows[k] < 1) return PGC_EINVAL;
+  if (d > (1 << 20)) return PGC_ENOTSUP;
+
+  pgc_ctx* ctx = new (std::nothrow) pgc_ctx();
+  if (!ctx) return PGC_ENOMEM;
+  ctx->n = n; ctx->s = s; ctx->c = s + 1; ctx->scheme = scheme; ctx->loss = loss; ctx->dtype = dtype;
+  ctx->d = d; ctx->K = K; ctx->lr = lr;
+  ctx->stream = static_cast<cudaStream_t>(stream);
+  ctx->esize = dtype == PGC_BF16 ? 2 : 4;
+  ctx->owners = scheme == PGC_FR ? n / ctx->c : n;
+  ctx->rows.assign(rows, rows + n);
+  ctx->row0.resize(n);
+  int64_t acc = 0;
+  for (int k = 0; k < n; ++k) { ctx->row0[k] = acc; acc += rows[k]; }
+  ctx->total_rows = acc;
+
+  if (loss != PGC_SOFTMAX) {
+    ctx->variant = grad_rows_variant(dtype, d, &ctx->ld);
+    if (ctx->variant < 0) { delete ctx; return PGC_ENOTSUP; }
+  } else {
+    ctx->ld = (int64_t)align_up((size_t)d, 64);
+  }
+  ctx->P = ctx->K * ctx->ld;
+  ctx->Kpad = (int64_t)align_up((size_t)K, 4);
+
+  cudaError_t e = cudaGetDevice(&ctx->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, ctx->device);
+  if (e != cudaSuccess) { delete ctx; return PGC_ECUDA; }
+
+  // phases and their tables
+  ctx->phases.resize(1 + ctx->c);
+  build_phase(ctx, ctx->phases[0], -1);
+  for (int o = 0; o < ctx->c; ++o) build_phase(ctx, ctx->phases[1 + o], o);
+  size_t max_partials = 0;
+  int64_t max_z = 0;
+  for (auto& ph : ctx->phases) {
+    const size_t np = ctx->loss == PGC_SOFTMAX ? ph.parts.size() * (size_t)ctx->P : ph.items.size() * (size_t)ctx->ld;
+    max_partials = std::max(max_partials, np);
+    max_z = std::max(max_z, ph.z_total);
+  }
+  std::vector<uint8_t> tab;
+  size_t off = 0;
+  std::vector<size_t> offs;
+  for (auto& ph : ctx->phases) {
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_scale);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_dest);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_row0);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_rows);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_zrow0);
+  }
+  // loss chunks (softmax): {row0, rows, 0} per chunk
+  std::vector<int64_t> ldesc;
+  if (loss == PGC_SOFTMAX) {
+    ctx->loss_chunk = std::min<int64_t>(ctx->total_rows, 32768);
+    for (int64_t r0 = 0; r0 < ctx->total_rows; r0 += ctx->loss_chunk) {
+      ldesc.push_back(r0);
+      ldesc.push_back(std::min(ctx->loss_chunk, ctx->total_rows - r0));
+      ldesc.push_back(0);
+    }
+  }
+  const size_t ldesc_off = align_up(off, 16);
+  put(tab, off, ldesc);
+  if (tab.empty()) tab.resize(16);
+
+  auto fail = [&](cudaError_t err) {
+    free_all(ctx);
+    delete ctx;
+    return err == cudaErrorMemoryAllocation ? PGC_ENOMEM : PGC_ECUDA;
+  };
+#define PGC_ALLOC(ptr, bytes)                                              \
+  do {                                                                     \
+    cudaError_t _e = cudaMalloc((void**)&(ptr), std::max<size_t>((bytes), 16)); \
+    if (_e != cudaSuccess) return fail(_e);                                \
+  } while (0)
+
+  const size_t Pb = (size_t)ctx->P * sizeof(float);
+  PGC_ALLOC(ctx->X, (size_t)ctx->total_rows * ctx->ld * ctx->esize);
+  PGC_ALLOC(ctx->y, (size_t)ctx->total_rows * 4);
+  PGC_ALLOC(ctx->w, Pb);
+  if (dtype == PGC_BF16) PGC_ALLOC(ctx->wb, (size_t)ctx->P * 2);
+  PGC_ALLOC(ctx->store, (size_t)ctx->owners * ctx->c * Pb);
+  PGC_ALLOC(ctx->U, (size_t)ctx->c * Pb);
+  PGC_ALLOC(ctx->gout, Pb);
+  PGC_ALLOC(ctx->partials, max_partials * sizeof(float));
+  if (loss == PGC_SOFTMAX)
+    PGC_ALLOC(ctx->Z, (size_t)std::max<int64_t>(max_z, ctx->loss_chunk) * ctx->Kpad * sizeof(float));
+  PGC_ALLOC(ctx->coeff, (size_t)n * sizeof(float));
+  PGC_ALLOC(ctx->status, sizeof(int));
+  PGC_ALLOC(ctx->loss_blocks, (size_t)ctx->loss_nblocks * sizeof(double));
+  PGC_ALLOC(ctx->loss_out, sizeof(double));
+  PGC_ALLOC(ctx->tables, tab.size());
+
+  cudaStream_t st = ctx->stream;
+  e = cudaMemcpyAsync(ctx->tables, tab.data(), tab.size(), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->X, 0, (size_t)ctx->total_rows * ctx->ld * ctx->esize, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->w, 0, Pb, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->store, 0, (size_t)ctx->owners * ctx->c * Pb, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->U, 0, (size_t)ctx->c * Pb, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->gout, 0, Pb, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->coeff, 0, (size_t)n * sizeof(float), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->status, 0, sizeof(int), st);
+  if (e == cudaSuccess && w0)
+    e = cudaMemcpy2DAsync(ctx->w, ctx->ld * sizeof(float), w0, d * sizeof(float), d * sizeof(float), K,
+                          cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && ctx->wb) e = launch_f32_to_bf16(ctx->w, ctx->wb, ctx->P, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return fail(e);
+
+  uint8_t* base = static_cast<uint8_t*>(ctx->tables);
+  for (size_t i = 0; i < ctx->phases.size(); ++i) {
+    Phase& ph = ctx->phases[i];
+    ph.d_items = reinterpret_cast<WorkItem*>(base + offs[7 * i + 0]);
+    ph.d_e_item0 = reinterpret_cast<int32_t*>(base + offs[7 * i + 1]);
+    ph.d_e_scale = reinterpret_cast<float*>(base + offs[7 * i + 2]);
+    ph.d_e_dest = reinterpret_cast<int32_t*>(base + offs[7 * i + 3]);
+    ph.d_e_row0 = reinterpret_cast<int64_t*>(base + offs[7 * i + 4]);
+    ph.d_e_rows = reinterpret_cast<int64_t*>(base + offs[7 * i + 5]);
+    ph.d_e_zrow0 = reinterpret_cast<int64_t*>(base + offs[7 * i + 6]);
+  }
+  ctx->loss_desc = nullptr;
+  if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
+#undef PGC_ALLOC
+  *out = ctx;
+  return PGC_OK;
+}
+
+int pgc_destroy(pgc_ctx* ctx) {
+  if (!ctx) return PGC_OK;
+  cudaStreamSynchronize(ctx->stream);
+  // loss_desc points into tables; do not free it twice
+  ctx->loss_desc = nullptr;
+  free_all(ctx);
+  delete ctx;
+  return PGC_OK;
+}
+
+int pgc_load_partitions(pgc_ctx* ctx, const void* const* X, const void* const* y, int32_t on_device) {
+  if (!ctx || !X || !y) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  for (int k = 0; k < ctx->n; ++k)
+    if (!X[k] || !y[k]) return PGC_EINVAL;
+  const cudaMemcpyKind kx = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+  const size_t es = ctx->esize;
+  for (int k = 0; k < ctx->n; ++k) {
+    uint8_t* dst = static_cast<uint8_t*>(ctx->X) + (size_t)ctx->row0[k] * ctx->ld * es;
+    PGC_CK(ctx, cudaMemcpy2DAsync(dst, ctx->ld * es, X[k], ctx->d * es, ctx->d * es, ctx->rows[k], kx, ctx->stream));
+    PGC_CK(ctx, cudaMemcpyAsync(static_cast<uint8_t*>(ctx->y) + (size_t)ctx->row0[k] * 4, y[k],
+                                (size_t)ctx->rows[k] * 4, kx, ctx->stream));
+  }
+  PGC_CK(ctx, cudaStreamSynchronize(ctx->stream));
+  ctx->loaded = true;
+  return PGC_OK;
+}
+
+int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, int32_t outputs_on_device,
+             pgc_step_info* info) {
+  if (!ctx || !mask) return PGC_EINVAL;
+  if (!ctx->loaded || ctx->broken) return PGC_ESTATE;
+  const int n = ctx->n, c = ctx->c;
+  MaskBits bits;
+  std::memset(&bits, 0, sizeof(bits));
+  int cnt = 0;
+  for (int i = 0; i < n; ++i) {
+    if (mask[i] > 1) return PGC_EMASK;
+    if (mask[i]) { bits.w[i >> 5] |= 1u << (i & 31); ++cnt; }
+  }
+  if (cnt != ctx->s) return PGC_EMASK;
+
+  const int64_t t = ctx->t;
+  const int pidx = t == 0 ? 0 : 1 + (int)((t - 1) % c);
+  Phase& ph = ctx->phases[pidx];
+  cudaStream_t st = ctx->stream;
+
+  PGC_CK(ctx, record_event(ctx));
+  int64_t nl[PGC_NKGROUPS] = {0, 1, 1};
+  // K1 / softmax gradient -> partials
+  if (ctx->loss != PGC_SOFTMAX) {
+    nl[PGC_KGRAD] = ph.items.empty() ? 0 : 1;
+    GradRowsArgs g;
+    g.loss = ctx->loss; g.dtype = ctx->dtype; g.d = ctx->d; g.ld = ctx->ld;
+    g.X = ctx->X; g.y = static_cast<const float*>(ctx->y); g.w = ctx->w;
+    g.items = ph.d_items; g.nitems = (int)ph.items.size(); g.max_item_rows = ph.max_item_rows;
+    g.partials = ctx->partials; g.status = ctx->status;
+    PGC_CK(ctx, launch_grad_rows(g, ctx->variant, st));
+  } else {
+    SoftmaxCCArgs a;
+    a.dtype = ctx->dtype; a.ld = ctx->ld; a.K = ctx->K; a.X = ctx->X; a.y = static_cast<const int32_t*>(ctx->y);
+    a.W = ctx->w; a.e_row0 = ph.d_e_row0; a.e_rows = ph.d_e_rows; a.e_zrow0 = ph.d_e_zrow0;
+    a.nE = (int)ph.parts.size(); a.max_rows = ph.max_rows; a.z_total = ph.z_total; a.Z = ctx->Z;
+    a.Kpad = ctx->Kpad; a.partials = ctx->partials;
+    nl[PGC_KGRAD] = 3;
+    PGC_CK(ctx, launch_softmax_cc(a, st));
+  }
+  PGC_CK(ctx, record_event(ctx));
+  // K4 commit into the stores
+  CommitArgs cm;
+  cm.partials = ctx->partials; cm.P = ctx->P; cm.e_item0 = ph.d_e_item0; cm.e_scale = ph.d_e_scale;
+  cm.e_dest = ph.d_e_dest; cm.ndest = ph.ndest; cm.nE = (int)ph.parts.size(); cm.store = ctx->store;
+  PGC_CK(ctx, launch_commit(cm, st));
+  PGC_CK(ctx, record_event(ctx));
+  // K5+K6 decode + SGD
+  DecodeArgs dc;
+  dc.scheme = ctx->scheme; dc.n = n; dc.s = ctx->s; dc.c = c; dc.slot = ph.slot; dc.owners = ctx->owners;
+  dc.mask = bits; dc.P = ctx->P; dc.store = ctx->store; dc.U = ctx->U; dc.w = ctx->w; dc.wb = ctx->wb;
+  dc.gout = ctx->gout; dc.lr = ctx->lr; dc.coeff_out = ctx->coeff; dc.status = ctx->status;
+  PGC_CK(ctx, launch_decode(dc, st));
+  PGC_CK(ctx, record_event(ctx));
+  if (ctx->timing) {
+    for (int k = 0; k < PGC_NKGROUPS; ++k) ctx->launches[k] += nl[k];
+    ++ctx->timed_steps;
+  }
+
+  if (grad_out) { int rc = copy_out(ctx, grad_out, ctx->gout, outputs_on_device); if (rc) return rc; }
+  if (w_out) { int rc = copy_out(ctx, w_out, ctx->w, outputs_on_device); if (rc) return rc; }
+  if (!outputs_on_device && (grad_out || w_out)) {
+    const int rc = read_status(ctx);
+    if (rc) return rc;
+  }
+  if (info) {
+    info->t = t;
+    info->slot = ph.slot;
+    info->received = n - ctx->s;
+    if (info->eval_partition)
+      for (int i = 0; i < n; ++i) info->eval_partition[i] = ph.slot < 0 ? -1 : held(ctx->scheme, n, c, i, ph.slot);
+    if (info->fr_rep && ctx->scheme == PGC_FR)
+      for (int g = 0; g < n / c; ++g) {
+        int rep = -1;
+        for (int l = 0; l < c && rep < 0; ++l)
+          if (!mask[g * c + l]) rep = g * c + l;
+        info->fr_rep[g] = rep;
+      }
+  }
+  ctx->t = t + 1;
+  ctx->stepped = true;
+  return PGC_OK;
+}
+
+int pgc_sync(pgc_ctx* ctx) {
+  if (!ctx) return PGC_EINVAL;
+  return read_status(ctx);
+}
+
+int pgc_loss(pgc_ctx* ctx, double* loss_out) {
+  if (!ctx || !loss_out) return PGC_EINVAL;
+  if (!ctx->loaded || ctx->broken) return PGC_ESTATE;
+  LossArgs a;
+  a.loss = ctx->loss; a.dtype = ctx->dtype; a.ld = ctx->ld; a.K = ctx->K; a.rows = ctx->total_rows;
+  a.X = ctx->X; a.y = ctx->y; a.w = ctx->w; a.blocksum = ctx->loss_blocks; a.nblocks = ctx->loss_nblocks;
+  a.out = ctx->loss_out; a.Z = ctx->Z; a.Kpad = ctx->Kpad; a.z_chunk_rows = ctx->loss_chunk;
+  a.chunk_desc = ctx->loss_desc;
+  PGC_CK(ctx, launch_loss(a, ctx->stream));
+  PGC_CK(ctx, cudaMemcpyAsync(loss_out, ctx->loss_out, sizeof(double), cudaMemcpyDeviceToHost, ctx->stream));
+  return read_status(ctx);
+}
+
+int pgc_get_store(pgc_ctx* ctx, int32_t worker, int32_t slot, float* out) {
+  if (!ctx || !out || worker < 0 || worker >= ctx->n || slot < 0 || slot >= ctx->c) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  const int owner = ctx->scheme == PGC_FR ? worker / ctx->c : worker;
+  const float* src = ctx->store + ((size_t)owner * ctx->c + slot) * ctx->P;
+  int rc = copy_out(ctx, out, src, 0);
+  if (rc) return rc;
+  return read_status(ctx);
+}
+
+int pgc_get_decode(pgc_ctx* ctx, float* coeff) {
+  if (!ctx || !coeff) return PGC_EINVAL;
+  if (!ctx->stepped || ctx->broken) return PGC_ESTATE;
+  PGC_CK(ctx, cudaMemcpyAsync(coeff, ctx->coeff, (size_t)ctx->n * sizeof(float), cudaMemcpyDeviceToHost, ctx->stream));
+  return read_status(ctx);
+}
+
+int pgc_get_weights(pgc_ctx* ctx, float* out) {
+  if (!ctx || !out) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  int rc = copy_out(ctx, out, ctx->w, 0);
+  if (rc) return rc;
+  return read_status(ctx);
+}
+
+int pgc_set_weights(pgc_ctx* ctx, const float* w) {
+  if (!ctx || !w) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  PGC_CK(ctx, cudaMemcpy2DAsync(ctx->w, ctx->ld * sizeof(float), w, ctx->d * sizeof(float), ctx->d * sizeof(float),
+                                ctx->K, cudaMemcpyHostToDevice, ctx->stream));
+  if (ctx->wb) PGC_CK(ctx, launch_f32_to_bf16(ctx->w, ctx->wb, ctx->P, ctx->stream));
+  return read_status(ctx);
+}
+
+int64_t pgc_step_count(const pgc_ctx* ctx) { return ctx ? ctx->t : -1; }
+
+int pgc_timing(pgc_ctx* ctx, int32_t enable) {
+  if (!ctx) return PGC_EINVAL;
+  PGC_CK(ctx, cudaStreamSynchronize(ctx->stream));
+  ctx->timing = enable != 0;
+  if (enable) {
+    ctx->ev_used = 0;
+    ctx->timed_steps = 0;
+    for (int k = 0; k < PGC_NKGROUPS; ++k) ctx->launches[k] = 0;
+  }
+  return PGC_OK;
+}
+
+int pgc_timing_read(pgc_ctx* ctx, double* ms, int64_t* launches, int64_t* steps_out) {
+  if (!ctx) return PGC_EINVAL;
+  PGC_CK(ctx, cudaStreamSynchronize(ctx->stream));
+  double acc[PGC_NKGROUPS] = {0, 0, 0};
+  // four events per recorded step: before grad, after grad, after commit, after decode
+  for (size_t i = 0; i + 3 < ctx->ev_used; i += 4) {
+    for (int k = 0; k < PGC_NKGROUPS; ++k) {
+      float t = 0.f;
+      PGC_CK(ctx, cudaEventElapsedTime(&t, ctx->ev_pool[i + k], ctx->ev_pool[i + k + 1]));
+      acc[k] += t;
+    }
+  }
+  if (ms)
+    for (int k = 0; k < PGC_NKGROUPS; ++k) ms[k] = acc[k];
+  if (launches)
+    for (int k = 0; k < PGC_NKGROUPS; ++k) launches[k] = ctx->launches[k];
+  if (steps_out) *steps_out = ctx->timed_steps;
+  return read_status(ctx);
+}
+
+}  // extern "C"

@@ -1,0 +1,130 @@
+// Internal interfaces between the host control code (pgc_api.cu) and the
+// kernel files.  Nothing here is part of the public ABI.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace pgc {
+
+// Error bits written to a context's device status word.
+enum : int {
+  kErrWaitTimeout = 1,   // a bounded mbarrier wait gave up
+  kErrBadMask = 2,       // the decode kernel saw a mask with popcount != s
+  kErrBadShape = 4,      // a kernel was launched with an impossible shape
+};
+
+// A contiguous row range of one evaluated partition, processed by one CTA.
+// Rows are global row indices into the packed feature buffer (all partitions
+// back to back, each row padded to `ld` elements).
+struct WorkItem {
+  int32_t e;        // position of the partition in the phase's evaluated list
+  int32_t part;     // partition index k
+  int64_t row0;     // first global row
+  int64_t rows;     // number of rows (>= 1)
+};
+
+// ---- K1: streaming gradient of logistic / least-squares partitions -------
+// For every work item: partial[item][0:ld] = sum over its rows x of
+// residual(x) * x, residual = sigmoid(x.w) - y (logistic) or x.w - y (lsq).
+struct GradRowsArgs {
+  int loss;                 // PGC_LOGISTIC or PGC_LSQ
+  int dtype;                // PGC_F32 or PGC_BF16
+  int64_t d, ld;            // features, padded row length (elements)
+  const void* X;            // packed features [total_rows][ld]
+  const float* y;           // packed labels [total_rows]
+  const float* w;           // parameters [ld] (padding is zero)
+  const WorkItem* items;    // device [nitems]
+  int nitems;
+  int max_item_rows;        // rows of the largest item (<= 8192)
+  float* partials;          // [nitems][ld]
+  int* status;              // device status word (error bits)
+};
+int grad_rows_variant(int dtype, int64_t d, int64_t* ld_out);  // chooses ld, returns variant id
+int grad_rows_stage_rows(int variant, int64_t ld, int dtype);
+cudaError_t launch_grad_rows(const GradRowsArgs& a, int variant, cudaStream_t st);
+
+// ---- K4: partial reduction + store commit ----------------------------------
+// For each evaluated partition e (CSR over items): g = scale[e] * sum of its
+// items' partials (in item order), written to every destination store
+// dest[e*ndest + j] (an index owner*c + slot, or -1 for none).
+struct CommitArgs {
+  const float* partials;    // [nitems][P]
+  int64_t P;                // floats per gradient (K * ld), multiple of 4
+  const int32_t* e_item0;   // [nE + 1]
+  const float* e_scale;     // [nE] 1 / m_e
+  const int32_t* e_dest;    // [nE * ndest]
+  int ndest;
+  int nE;
+  float* store;             // [owners * c][P]
+};
+cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st);
+
+// ---- K5 + K6: decode coefficients from the mask, decode, SGD --------------
+constexpr int kMaxWorkers = 1024;
+struct MaskBits {
+  uint32_t w[kMaxWorkers / 32];
+};
+struct DecodeArgs {
+  int scheme, n, s, c;
+  int slot;                 // o_t refreshed this step, or -1: all slots (warm-up)
+  int owners;               // stores: n (CR) or n / c (FR groups)
+  MaskBits mask;            // bit i = 1: worker i straggles
+  int64_t P;                // floats per gradient (multiple of 4)
+  float* store;             // [owners * c][P]
+  float* U;                 // [c][P] slot totals
+  float* w;                 // [P] parameters, updated in place
+  uint16_t* wb;             // [P] bf16 copy of w, or nullptr
+  float* gout;              // [P] decoded gradient
+  float lr;
+  float* coeff_out;         // [n] per-worker coefficient a_i (written by CTA 0)
+  int* status;
+};
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
+
+// ---- generic softmax gradient on CUDA cores --------------------------------
+// logits Z[r][k] = sum_j W[k][j] x_r[j] for the rows of each evaluated
+// partition, then R = softmax(Z) - onehot(y) in place, then
+// partial[e][k*ld + j] = sum_{r in e} R[r][k] x_r[j].
+struct SoftmaxCCArgs {
+  int dtype;
+  int64_t ld, K;
+  const void* X;            // packed [total_rows][ld]
+  const int32_t* y;         // packed class labels
+  const float* W;           // [K][ld]
+  const int64_t* e_row0;    // [nE] global first row of each evaluated partition
+  const int64_t* e_rows;    // [nE]
+  const int64_t* e_zrow0;   // [nE] first row of the partition in Z
+  int nE;
+  int64_t max_rows;         // max rows of an evaluated partition
+  int64_t z_total;          // rows of Z (sum of the evaluated partitions' rows)
+  float* Z;                 // scratch [z_total][Kpad]
+  int64_t Kpad;
+  float* partials;          // [nE][K*ld]
+};
+cudaError_t launch_softmax_cc(const SoftmaxCCArgs& a, cudaStream_t st);
+
+// ---- full loss ------------------------------------------------------------
+// Per-row f summed in fp64 into blocksum[block]; a second pass adds them in
+// block order.
+struct LossArgs {
+  int loss, dtype;
+  int64_t ld, K, rows;      // all rows of all partitions
+  const void* X;
+  const void* y;            // float (logistic/lsq) or int32 (softmax)
+  const float* w;           // [K][ld]
+  double* blocksum;         // scratch [nblocks]
+  int nblocks;
+  double* out;              // device double
+  // softmax only: logits are formed in row chunks
+  float* Z;                 // scratch [z_chunk_rows][Kpad]
+  int64_t Kpad;
+  int64_t z_chunk_rows;
+  const int64_t* chunk_desc; // device [3 * nchunks]: {row0, rows, 0} per chunk
+};
+cudaError_t launch_loss(const LossArgs& a, cudaStream_t st);
+
+// ---- misc -------------------------------------------------------------------
+cudaError_t launch_f32_to_bf16(const float* src, uint16_t* dst, int64_t count, cudaStream_t st);
+
+}  // namespace pgc

@@ -16,3 +16,21 @@ def pytest_configure(config):
 @pytest.fixture(scope="session")
 def root_dir():
     return ROOT
+
+
+@pytest.fixture(scope="session")
+def libpgc():
+    """The built library (built here if missing; nvcc cross-compiles without a GPU)."""
+    from paper_2607_20739_gb300 import build as B
+    B.build()
+    from paper_2607_20739_gb300 import binding
+    return binding
+
+
+@pytest.fixture(scope="session")
+def cuda(libpgc):
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("GPU test collected on a machine without CUDA")
+    torch.cuda.init()
+    return torch
