@@ -34,6 +34,8 @@ extern "C" {
 #define PGC_ECUDA    (-5)  /* a CUDA runtime call or kernel failed           */
 #define PGC_ENOTSUP  (-6)  /* valid but unsupported combination             */
 #define PGC_ETIMEOUT (-7)  /* a bounded device-side wait gave up            */
+#define PGC_ESCRATCH (-8)  /* problem larger than pgc_gradient_noalloc's
+                              fixed scratch                                 */
 
 /* ---- enumerations (passed as int32) ------------------------------------ */
 /* Dataset placement, §III: FR needs c | n; CR places cyclically.          */
@@ -206,6 +208,40 @@ int pgc_timing(pgc_ctx *ctx, int32_t enable);
  * *steps_out (nullable) receives the number of recorded steps.
  */
 int pgc_timing_read(pgc_ctx *ctx, double *ms, int64_t *launches, int64_t *steps_out);
+
+/* ---- allocation-free gradient --------------------------------------------- */
+
+/*
+ * pgc_gradient_noalloc — g_out = (1/m) sum over the m rows x of one partition
+ * of r(x) * x, with r = sigmoid(x.w) - y (PGC_LOGISTIC) or x.w - y (PGC_LSQ):
+ * the per-partition gradient pgc_step evaluates, computed without allocating
+ * any device memory.  The paper has no counterpart; this exists for callers
+ * that cannot call cudaMalloc / cudaFree when they need a gradient: a
+ * framework whose caching pool already holds the free device memory, or a
+ * loop that must not take cudaFree's implicit device synchronisation.
+ *
+ *   X     : device [m][d] features (PGC_F32, or PGC_BF16 bits), 16-byte aligned
+ *   y     : device [m] float32 labels;  w: device [d] float32 parameters
+ *   g_out : device [d] float32, 16-byte aligned (written)
+ *   stream: cudaStream_t to run on; the call waits for it before returning.
+ *
+ * Scratch: a fixed 16 MiB array inside the library (a __device__ global),
+ * held on every GPU that loads the library until the process exits.  The
+ * first call on a device looks up the array's device address (with that
+ * device current); make that first call before any stream capture.  All
+ * calls share the array and it keeps the last call's contents; each call
+ * rewrites what it reads, but calls that overlap on the GPU (other streams,
+ * other threads) race on it.
+ *
+ * Limits: d must be a row length the gradient kernel takes without padding
+ * (fp32: 32, 64, 128 * 2^k up to 16384; bf16: 64, 128, 256 * 2^k up to
+ * 32768), else PGC_ENOTSUP.  Partial sums need ceil(m / 8192) * 4 d bytes or
+ * more; problems that do not fit the 16 MiB return PGC_ESCRATCH (fp32 d =
+ * 16384 fits up to about two million rows).  Other errors: PGC_EINVAL,
+ * PGC_ECUDA, PGC_ETIMEOUT.
+ */
+int pgc_gradient_noalloc(int32_t loss, int32_t dtype, int64_t m, int64_t d, const void *X,
+                         const float *y, const float *w, float *g_out, void *stream);
 
 #ifdef __cplusplus
 }

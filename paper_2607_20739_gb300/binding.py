@@ -24,7 +24,7 @@ if not os.path.exists(LIB_PATH):
 
 lib = C.CDLL(LIB_PATH)
 
-OK, EINVAL, EMASK, ESTATE, ENOMEM, ECUDA, ENOTSUP, ETIMEOUT = 0, -1, -2, -3, -4, -5, -6, -7
+OK, EINVAL, EMASK, ESTATE, ENOMEM, ECUDA, ENOTSUP, ETIMEOUT, ESCRATCH = 0, -1, -2, -3, -4, -5, -6, -7, -8
 FR, CR = 0, 1
 LOGISTIC, LSQ, SOFTMAX = 0, 1, 2
 F32, BF16 = 0, 1
@@ -60,6 +60,7 @@ _sig = {
     "pgc_step_count": (C.c_int64, [_vp]),
     "pgc_timing": (C.c_int, [_vp, _i32]),
     "pgc_timing_read": (C.c_int, [_vp, C.POINTER(C.c_double), C.POINTER(_i64), C.POINTER(_i64)]),
+    "pgc_gradient_noalloc": (C.c_int, [_i32, _i32, _i64, _i64, _vp, _vp, _vp, _vp, _vp]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(lib, _name)

@@ -259,6 +259,7 @@ const char* pgc_strerror(int32_t code) {
     case PGC_ECUDA: return "CUDA error";
     case PGC_ENOTSUP: return "unsupported combination";
     case PGC_ETIMEOUT: return "a bounded device-side wait timed out";
+    case PGC_ESCRATCH: return "problem too large for the fixed scratch of pgc_gradient_noalloc";
     default: return "unknown status";
   }
 }

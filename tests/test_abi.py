@@ -27,7 +27,7 @@ def test_every_declared_symbol_is_exported(libpgc, root_dir):
 
 
 def test_strerror_covers_codes(libpgc):
-    for code in range(0, -8, -1):
+    for code in range(0, -9, -1):
         assert libpgc.lib.pgc_strerror(code)
     assert b"unknown" in libpgc.lib.pgc_strerror(-99)
 
