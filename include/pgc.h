@@ -235,9 +235,10 @@ int pgc_timing_read(pgc_ctx *ctx, double *ms, int64_t *launches, int64_t *steps_
  *
  * Limits: d must be a row length the gradient kernel takes without padding
  * (fp32: 32, 64, 128 * 2^k up to 16384; bf16: 64, 128, 256 * 2^k up to
- * 32768), else PGC_ENOTSUP.  Partial sums need ceil(m / 8192) * 4 d bytes or
- * more; problems that do not fit the 16 MiB return PGC_ESCRATCH (fp32 d =
- * 16384 fits up to about two million rows).  Other errors: PGC_EINVAL,
+ * 32768), else PGC_ENOTSUP.  The scratch holds a copy of the m labels (4 m
+ * bytes) and one partial sum of 4 d bytes per SM; problems that do not fit
+ * the 16 MiB return PGC_ESCRATCH (on a 152-SM GPU: about 1.7 million rows at
+ * fp32 d = 16384, about 4 million at d = 1024).  Other errors: PGC_EINVAL,
  * PGC_ECUDA, PGC_ETIMEOUT.
  */
 int pgc_gradient_noalloc(int32_t loss, int32_t dtype, int64_t m, int64_t d, const void *X,

@@ -1,268 +1,477 @@
 // K1 — per-partition gradient of logistic and least-squares losses, one pass
 // over the features (§III: g_k = (1/m_k) sum_{x in D_k} grad f; the 1/m_k is
-// applied by the commit kernel).
+// applied when the partition is committed).
 //
-// Each CTA streams one work item (a contiguous row range of one partition)
-// from HBM into shared memory with 1-D bulk async copies (one producer
-// thread, a ring of S stages, mbarrier full/empty handshakes).  Every row is
-// read from HBM once: it is dotted with w, turned into the residual
-// r = sigmoid(x.w) - y (logistic) or x.w - y (least squares), and
-// accumulated as r * x, all while it sits in shared memory.
+// Work: the evaluated partitions' rows are cut into work items (contiguous
+// row ranges of one partition).  A persistent grid (at most one CTA per SM)
+// takes items dynamically: item blockIdx.x first, then the next free index
+// from a device counter, so SMs that stream faster take more items.  Each
+// item's sum over its rows of r(x) * x goes to its own partial slot, so the
+// result does not depend on which CTA took which item.
 //
+// Per CTA: one producer thread streams each item's rows from HBM into a ring
+// of S shared-memory stages with 1-D bulk async copies (rows and their labels,
+// completion counted on the stage's mbarrier); 8 consumer warps dot each row
+// with w, form the residual r = sigmoid(x.w) - y (logistic) or x.w - y (least
+// squares) and accumulate r * x while the row sits in shared memory, so every
+// feature byte is read from HBM once.
 //   warp-row  (row <= 1024 fp32 / 2048 bf16 elements): one warp per row; each
 //             lane holds NCH chunks of VEC elements of the row, of w and of
-//             its gradient accumulator; the dot is a warp-shuffle sum.  The
-//             8 warps' accumulators are summed in a fixed order at the end.
-//   block-row (longer rows): all 256 consumer threads share each row; each
-//             thread owns NCH chunks of columns; the dot is a shuffle sum
-//             plus one shared-memory exchange per stage.
+//             its accumulator; the dot is a warp-shuffle sum; at the end of an
+//             item the 8 warps' accumulators are summed in a fixed order.
+//   block-row (longer rows): the 256 consumer threads share each row; each
+//             owns NCH chunks of columns; the dots of a stage are exchanged
+//             once through shared memory.
 //
-// Output: partial[item][0:ld] = sum over the item's rows of r * x (fp32).
-#include "dev_common.cuh"
-#include "pgc_internal.h"
-#include "../../include/pgc.h"
+// Item ends: consumers hand their accumulators to a tail warp (through a
+// shared buffer and two mbarriers) and keep streaming.  The tail warp sums the
+// 8 warps' accumulators in a fixed order into the item's partial slot and,
+// with tail >= 1, counts the item for its partition.  When that count
+// completes a partition, the consumers commit it at their next item end (or
+// after their last item): ordered sum of the partition's partials, scaled by
+// 1/m, into its destination stores.  With tail == 2 the CTA that commits the
+// last partition also derives the decode coefficients from the mask, decodes
+// and applies the SGD update.
+//
+// Programmatic dependent launch: the producer streams its first item before
+// waiting for the previous step's kernel; consumers wait before reading w.
+//
+// Every wait is bounded (mbarrier try_wait with an iteration and time limit).
+// Consumer warps synchronise through mbarriers, never named barriers, so a
+// wait that gives up cannot leave another warp blocked: the CTA then skips
+// its remaining work, flags the status word and exits.
+#include "tail.cuh"
 
 namespace pgc {
 
 constexpr int kNW = 8;                 // consumer warps per CTA
 constexpr int kNT = kNW * 32;          // consumer threads
-constexpr int kThreads = kNT + 32;     // + one producer warp
-constexpr int kMaxItemRows = 8192;     // labels of one item staged in smem
+constexpr int kThreads = kNT + 64;     // + a producer warp + a tail warp
+constexpr int kProducer = kNT;        // producer thread
+constexpr int kTailWarp = kNW + 1;     // warp index of the tail warp
+
+struct StageHdr {
+  int item;      // work item, or -1: no more work
+  int e;         // evaluated-partition position of the item
+  int rows;      // rows in this stage
+  int lab_off;   // index of the stage's first label in its label slot
+  int last;      // last stage of the item
+  int pad[3];
+};
 
 struct StageCfg {
-  int SR;            // rows per stage
-  int S;             // stages
+  int SR;              // rows per stage
+  int S;               // stages
   uint32_t stage_bytes;
-  size_t smem;       // dynamic shared memory
+  int LS;              // floats per label slot
+  size_t red_bytes;    // item-end reduction buffer
+  size_t plan_bytes;   // decode plan (fused decode only)
+  size_t smem;         // dynamic shared memory
 };
 
 __device__ __forceinline__ float residual(int loss, float z, float y) {
   return loss == PGC_LOGISTIC ? 1.0f / (1.0f + expf(-z)) - y : z - y;
 }
 
-// Shared-memory map: [2S mbarriers | labels | (block-row: dot exchange) | stages]
-struct SmemMap {
+// Item handoff between the consumers and the tail warp.
+struct Handoff {
+  int item;            // item whose accumulators are in red, or -1: no more items
+  int e;
+  int commit;          // set by the tail warp: partition to commit, or -1
+  int decode;          // set by the consumers: this CTA decodes
+};
+
+// Shared memory: [full S | empty S | sync, red_full, red_free, tail_done]
+//                [handoff] [S headers] [S label slots] [red / decode scratch]
+//                [dot exchange] [S stages]
+struct Smem {
   uint64_t* full;
   uint64_t* empty;
-  float* ylab;
+  uint64_t* sync;       // consumer barrier (count kNW)
+  uint64_t* red_full;   // consumers -> tail warp (count kNW)
+  uint64_t* red_free;   // tail warp -> consumers (count 1)
+  Handoff* ho;
+  DecodePlan* plan;     // decode coefficients (tail == 2), derived at kernel start
+  StageHdr* hdr;
+  float* lab;
+  uint8_t* red;
   float* xdot;
   uint8_t* stages;
 };
 
-__device__ __forceinline__ SmemMap carve(uint8_t* smem, int S, int max_rows, int SR, bool block_row) {
-  SmemMap m;
-  m.full = reinterpret_cast<uint64_t*>(smem);
-  m.empty = m.full + S;
-  size_t off = 128;
-  m.ylab = reinterpret_cast<float*>(smem + off);
-  off += ((size_t)max_rows * 4 + 127) & ~size_t(127);
-  m.xdot = reinterpret_cast<float*>(smem + off);
-  if (block_row) off += ((size_t)2 * SR * kNW * 4 + 127) & ~size_t(127);
-  m.stages = smem + off;
+__host__ __device__ inline size_t a128(size_t v) { return (v + 127) & ~size_t(127); }
+
+__host__ __device__ inline size_t fixed_bytes(int S, int LS, size_t red, int SR, bool block_row, size_t plan) {
+  return a128(sizeof(uint64_t) * (2 * S + 4)) + a128(sizeof(Handoff)) + a128(plan) + a128(sizeof(StageHdr) * S) +
+         a128(sizeof(float) * LS * S) + a128(red) + (block_row ? a128(sizeof(float) * 2 * SR * kNW) : 0);
+}
+
+__device__ __forceinline__ Smem carve(uint8_t* base, const StageCfg& c, bool block_row) {
+  Smem m;
+  size_t off = 0;
+  m.full = reinterpret_cast<uint64_t*>(base);
+  m.empty = m.full + c.S;
+  m.sync = m.empty + c.S;
+  m.red_full = m.sync + 1;
+  m.red_free = m.sync + 2;
+  off = a128(sizeof(uint64_t) * (2 * c.S + 4));
+  m.ho = reinterpret_cast<Handoff*>(base + off);
+  off = a128(off + sizeof(Handoff));
+  m.plan = reinterpret_cast<DecodePlan*>(base + off);
+  off = a128(off + c.plan_bytes);
+  m.hdr = reinterpret_cast<StageHdr*>(base + off);
+  off = a128(off + sizeof(StageHdr) * c.S);
+  m.lab = reinterpret_cast<float*>(base + off);
+  off = a128(off + sizeof(float) * c.LS * c.S);
+  m.red = base + off;
+  off = a128(off + c.red_bytes);
+  m.xdot = reinterpret_cast<float*>(base + off);
+  if (block_row) off = a128(off + sizeof(float) * 2 * c.SR * kNW);
+  m.stages = base + off;
   return m;
 }
 
-// Producer: stream `nst` stages of the item's rows; afterwards wait until
-// every issued copy has landed so no copy outlives the CTA.
-__device__ __forceinline__ void produce(const SmemMap& sm, const uint8_t* src, int64_t rows, int64_t rb,
-                                        int SR, int S, uint32_t stage_bytes, int* status) {
+// A barrier of the 8 consumer warps on an mbarrier (count kNW), bounded.
+struct ConsumerSync {
+  uint64_t* bar;
+  uint32_t phase;
+  int* status;
+  __device__ __forceinline__ bool operator()() {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+    const bool ok = mbar_wait(bar, phase, status);
+    phase ^= 1u;
+    return __all_sync(0xffffffffu, ok);
+  }
+};
+
+// ---------------------------------------------------------------------------
+// producer
+// ---------------------------------------------------------------------------
+__device__ void produce(const GradRowsArgs& a, const Smem& sm, const StageCfg& c, int64_t rb) {
   const uint64_t pol = policy_evict_first();
-  const int nst = (int)((rows + SR - 1) / SR);
-  int issued = 0;
-  for (int i = 0; i < nst; ++i) {
-    const int s = i % S;
-    if (i >= S && !mbar_wait(&sm.empty[s], ((i / S) - 1) & 1, status)) break;
-    const int64_t r = rows - (int64_t)i * SR < SR ? rows - (int64_t)i * SR : SR;
-    const uint32_t bytes = (uint32_t)(r * rb);
-    mbar_arrive_expect_tx(&sm.full[s], bytes);
-    bulk_g2s_stream(sm.stages + (size_t)s * stage_bytes, src + (size_t)i * SR * rb, bytes, &sm.full[s], pol);
-    issued = i + 1;
+  const uint8_t* X = static_cast<const uint8_t*>(a.X);
+  const uint8_t* Y = reinterpret_cast<const uint8_t*>(a.y);
+  int i = 0;                     // stages issued
+  bool ok = true, waited = false;
+  int item = blockIdx.x;
+  while (ok && item < a.nitems) {
+    const WorkItem it = a.items[item];
+    const int nst = (int)((it.rows + c.SR - 1) / c.SR);
+    for (int j = 0; j < nst; ++j) {
+      const int s = i % c.S;
+      if (i >= c.S && !mbar_wait(&sm.empty[s], ((i / c.S) - 1) & 1, a.status)) { ok = false; break; }
+      const int64_t r0 = it.row0 + (int64_t)j * c.SR;
+      const int rows = (int)(it.rows - (int64_t)j * c.SR < c.SR ? it.rows - (int64_t)j * c.SR : c.SR);
+      const int64_t la = r0 & ~int64_t(3);                      // 16-byte aligned label start
+      const uint32_t lbytes = (uint32_t)(((r0 + rows - la) * 4 + 15) & ~int64_t(15));
+      StageHdr h;
+      h.item = item; h.e = it.e; h.rows = rows; h.lab_off = (int)(r0 - la); h.last = j == nst - 1;
+      sm.hdr[s] = h;
+      const uint32_t xbytes = (uint32_t)(rows * rb);
+      mbar_arrive_expect_tx(&sm.full[s], xbytes + lbytes);
+      bulk_g2s_stream(sm.stages + (size_t)s * c.stage_bytes, X + r0 * rb, xbytes, &sm.full[s], pol);
+      bulk_g2s(sm.lab + (size_t)s * c.LS, Y + la * 4, lbytes, &sm.full[s]);
+      ++i;
+    }
+    if (!ok || !a.work_ctr) break;
+    if (a.pdl && !waited) { grid_dep_wait(); waited = true; }   // counters belong to the previous step until now
+    item = (int)gridDim.x + atomicAdd(a.work_ctr, 1);
   }
-  for (int s = 0; s < S && s < issued; ++s) {
-    const int last = ((issued - 1 - s) / S) * S + s;
-    mbar_wait(&sm.full[s], (last / S) & 1, status);
+  if (ok) {   // end marker: a stage without data
+    const int s = i % c.S;
+    if (i < c.S || mbar_wait(&sm.empty[s], ((i / c.S) - 1) & 1, a.status)) {
+      sm.hdr[s].item = -1;
+      mbar_arrive(&sm.full[s]);
+      ++i;
+    }
+  }
+  if (a.work_ctr) {
+    if (a.pdl && !waited) grid_dep_wait();
+    // the last producer to finish resets the item counter for the next step
+    if (atomicAdd(a.prod_done, 1) == (int)gridDim.x - 1) {
+      *a.work_ctr = 0;
+      *a.prod_done = 0;
+    }
+  }
+  // no copy may outlive the CTA: wait for the last use of every stage
+  for (int s = 0; s < c.S && s < i; ++s) {
+    const int last = ((i - 1 - s) / c.S) * c.S + s;
+    mbar_wait(&sm.full[s], (last / c.S) & 1, a.status);
   }
 }
 
+// ---------------------------------------------------------------------------
+// tail warp: per-item reduction and partition counting
+// ---------------------------------------------------------------------------
+__device__ void tail_warp(const GradRowsArgs& a, const Smem& sm, bool warp_row) {
+  const int lane = threadIdx.x & 31;
+  if (a.tail == 2) derive_plan_warp(a.dec, *sm.plan, lane);   // depends only on the mask
+  if (a.pdl) grid_dep_wait();          // partials and counters belong to the previous step until now
+  const float* red = reinterpret_cast<const float*>(sm.red);
+  for (uint32_t j = 0;; ++j) {
+    if (!__all_sync(0xffffffffu, mbar_wait(sm.red_full, j & 1u, a.status))) break;
+    const int item = sm.ho->item, e = sm.ho->e;
+    if (item < 0) break;
+    if (warp_row) {
+      // fixed-order sum of the 8 warps' accumulators into the item's partial
+      float4* out = reinterpret_cast<float4*>(a.partials + (size_t)item * a.ld);
+      const float4* r4 = reinterpret_cast<const float4*>(red);
+      const int64_t L4 = a.ld / 4;
+      for (int64_t q = lane; q < L4; q += 32) {
+        float4 acc = r4[q];
+#pragma unroll
+        for (int w8 = 1; w8 < kNW; ++w8) acc = f4add(acc, r4[(size_t)w8 * L4 + q]);
+        out[q] = acc;
+      }
+    }
+    int commit = -1;
+    if (a.tail) {
+      __syncwarp();
+      if (lane == 0) {
+        __threadfence();               // the item's partial (written by this warp or by the consumers)
+        const int prev = atomicAdd(&a.cnt_e[e], 1);
+        if (prev == a.e_item0[e + 1] - a.e_item0[e] - 1) {
+          a.cnt_e[e] = 0;              // every item of e has arrived: reset for the next step
+          __threadfence();             // acquire the other CTAs' partials before handing e to the consumers
+          commit = e;
+        }
+      }
+      commit = __shfl_sync(0xffffffffu, commit, 0);
+    }
+    if (lane == 0) {
+      sm.ho->commit = commit;
+      mbar_arrive(sm.red_free);
+    }
+    __syncwarp();
+  }
+}
+
+// Consumers: commit partition e (all 256 consumer threads), then count it;
+// the CTA completing the last partition decodes when tail == 2.
+__device__ void consumer_commit(const GradRowsArgs& a, const Smem& sm, int e, int tid, ConsumerSync& bar, bool& ok) {
+  // the tail warp acquired the other CTAs' partials (atomic + fence) before
+  // handing e over through red_free
+  commit_block(a.partials, a.ld, a.e_item0[e], a.e_item0[e + 1], a.e_scale[e], a.e_dest + (int64_t)e * a.ndest,
+               a.ndest, a.store, tid, kNT);
+  if (!bar()) { ok = false; return; }
+  if (tid == 0) {
+    __threadfence();                   // release the stores written by the whole CTA
+    const bool all = atomicAdd(a.cnt_all, 1) == a.nE - 1;
+    if (all) {
+      *a.cnt_all = 0;
+      __threadfence();                 // acquire the other committers' stores
+    }
+    if (all && a.tail == 2) sm.ho->decode = 1;
+  }
+}
+
+__device__ void consumer_decode(const GradRowsArgs& a, const Smem& sm, int tid) {
+  if (tid < 32) write_coeffs_warp(a.dec, tid);
+  decode_columns(a.dec, *sm.plan, tid, kNT);
+}
+
+// Item end, consumer side, called by all 8 warps at the same stage.
+// handover_begin: wait until the tail warp has taken the previous item (so
+// red and the handoff slot are free) and run the commit it asked for.
+__device__ __forceinline__ bool handover_begin(const GradRowsArgs& a, const Smem& sm, uint32_t ends, ConsumerSync& bar,
+                                               bool& ok) {
+  if (ends == 0) return true;
+  if (!__all_sync(0xffffffffu, mbar_wait(sm.red_free, (ends - 1) & 1u, a.status))) { ok = false; return false; }
+  const int ce = sm.ho->commit;          // written by the tail warp before red_free: same for every warp
+  if (ce >= 0) {
+    consumer_commit(a, sm, ce, (int)threadIdx.x, bar, ok);
+    if (!ok) return false;
+  }
+  return true;
+}
+
+// handover_end: publish the item (or -1: no more) to the tail warp.
+__device__ __forceinline__ void handover_end(const Smem& sm, int item, int e, uint32_t& ends) {
+  if (threadIdx.x == 0) { sm.ho->item = item; sm.ho->e = e; }
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(sm.red_full);
+  ++ends;
+}
+
+// After the last item: final handoff, pending commit, decode if this CTA
+// committed the last partition.
+__device__ __forceinline__ void consumers_finish(const GradRowsArgs& a, const Smem& sm, uint32_t& ends,
+                                                 ConsumerSync& bar, bool& ok) {
+  if (ok && handover_begin(a, sm, ends, bar, ok)) {
+    handover_end(sm, -1, -1, ends);
+    if (!bar()) ok = false;              // the decode flag is written before this barrier
+    if (ok && sm.ho->decode) consumer_decode(a, sm, (int)threadIdx.x);
+  } else if (threadIdx.x < kNT) {
+    // release the tail warp even on failure: it stops at item -1 or at its own bound
+    handover_end(sm, -1, -1, ends);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// consumers
+// ---------------------------------------------------------------------------
 template <typename T, int VEC, int NCH>
-__global__ void __launch_bounds__(kThreads, 1)
-grad_rows_warp(GradRowsArgs a, int SR, int S, uint32_t stage_bytes, int max_rows) {
-  extern __shared__ __align__(128) uint8_t smem[];
+__device__ void consume_warp_row(const GradRowsArgs& a, const Smem& sm, const StageCfg& c, int64_t rb) {
   using V = Vec<T, VEC>;
   constexpr int E = NCH * VEC;
-  const SmemMap sm = carve(smem, S, max_rows, SR, false);
-  const WorkItem it = a.items[blockIdx.x];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t rb = a.ld * (int64_t)sizeof(T);
-  const int nst = (int)((it.rows + SR - 1) / SR);
-  __shared__ int cta_err;
-
-  if (threadIdx.x == 0) {
-    cta_err = 0;
-    for (int s = 0; s < S; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kNW);
+  ConsumerSync bar{sm.sync, 0u, a.status};
+  if (a.pdl) grid_dep_wait();                       // w is the previous step's output
+  float wr[E], acc[E];
+#pragma unroll
+  for (int j = 0; j < NCH; ++j)
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+      wr[j * VEC + v] = a.w[(j * 32 + lane) * VEC + v];
+      acc[j * VEC + v] = 0.f;
     }
-    fence_mbar_init();
-  }
-  __syncthreads();
-
-  if (warp == kNW) {
-    if (lane == 0)
-      produce(sm, reinterpret_cast<const uint8_t*>(a.X) + it.row0 * rb, it.rows, rb, SR, S, stage_bytes,
-              a.status);
-  } else {
-    // labels of the whole item, and this lane's slice of w
-    for (int64_t r = threadIdx.x; r < it.rows; r += kNT) sm.ylab[r] = a.y[it.row0 + r];
-    float wr[E], acc[E];
+  float* red = reinterpret_cast<float*>(sm.red);
+  uint32_t ends = 0;
+  bool ok = true;
+  for (int i = 0; ok; ++i) {
+    const int s = i % c.S;
+    if (!__all_sync(0xffffffffu, mbar_wait(&sm.full[s], (i / c.S) & 1, a.status))) { ok = false; break; }
+    const StageHdr h = sm.hdr[s];
+    if (h.item < 0) break;
+    const uint8_t* st = sm.stages + (size_t)s * c.stage_bytes;
+    const float* lab = sm.lab + (size_t)s * c.LS + h.lab_off;
+    for (int rr = warp; rr < h.rows; rr += kNW) {
+      const typename V::raw* row = reinterpret_cast<const typename V::raw*>(st + rr * rb);
+      float x[E];
 #pragma unroll
-    for (int j = 0; j < NCH; ++j)
+      for (int j = 0; j < NCH; ++j) V::widen(row[j * 32 + lane], &x[j * VEC]);
+      float dot = 0.f;
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        wr[j * VEC + v] = a.w[(j * 32 + lane) * VEC + v];
-        acc[j * VEC + v] = 0.f;
-      }
-    named_bar_sync(1, kNT);
-    bool ok = true;
-    for (int i = 0; i < nst && ok; ++i) {
-      const int s = i % S;
-      const bool got = mbar_wait(&sm.full[s], (i / S) & 1, a.status);
-      if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
-      const int64_t rows_i = it.rows - (int64_t)i * SR < SR ? it.rows - (int64_t)i * SR : SR;
-      const uint8_t* st = sm.stages + (size_t)s * stage_bytes;
-      for (int rr = warp; rr < rows_i; rr += kNW) {
-        const typename V::raw* row = reinterpret_cast<const typename V::raw*>(st + rr * rb);
-        float x[E];
+      for (int k = 0; k < E; ++k) dot = fmaf(x[k], wr[k], dot);
+      dot = warp_sum(dot);
+      const float r = residual(a.loss, dot, lab[rr]);
 #pragma unroll
-        for (int j = 0; j < NCH; ++j) V::widen(row[j * 32 + lane], &x[j * VEC]);
-        float dot = 0.f;
-#pragma unroll
-        for (int e = 0; e < E; ++e) dot = fmaf(x[e], wr[e], dot);
-        dot = warp_sum(dot);
-        const float r = residual(a.loss, dot, sm.ylab[(int64_t)i * SR + rr]);
-#pragma unroll
-        for (int e = 0; e < E; ++e) acc[e] = fmaf(r, x[e], acc[e]);
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sm.empty[s]);
+      for (int k = 0; k < E; ++k) acc[k] = fmaf(r, x[k], acc[k]);
     }
-    if (!ok) atomicExch(&cta_err, 1);
-    named_bar_sync(1, kNT);
-    if (!cta_err) {
-      // every stage was consumed, so no copy is in flight: reuse the stages
-      float* red = reinterpret_cast<float*>(sm.stages);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sm.empty[s]);
+    if (h.last) {
+      if (!handover_begin(a, sm, ends, bar, ok)) break;
 #pragma unroll
       for (int j = 0; j < NCH; ++j)
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) red[(size_t)warp * a.ld + (j * 32 + lane) * VEC + v] = acc[j * VEC + v];
-      named_bar_sync(1, kNT);
-      float* out = a.partials + (size_t)blockIdx.x * a.ld;
-      for (int64_t col = threadIdx.x; col < a.ld; col += kNT) {
-        float sum = 0.f;
-#pragma unroll
-        for (int w8 = 0; w8 < kNW; ++w8) sum += red[(size_t)w8 * a.ld + col];
-        out[col] = sum;
-      }
+        for (int v = 0; v < VEC; ++v) {
+          red[(size_t)warp * a.ld + (j * 32 + lane) * VEC + v] = acc[j * VEC + v];
+          acc[j * VEC + v] = 0.f;
+        }
+      handover_end(sm, h.item, h.e, ends);
     }
   }
-  __syncthreads();
+  consumers_finish(a, sm, ends, bar, ok);
+  if (!ok) atomicOr(a.status, kErrWaitTimeout);
 }
 
 template <typename T, int VEC, int NCH>
-__global__ void __launch_bounds__(kThreads, 1)
-grad_rows_block(GradRowsArgs a, int SR, int S, uint32_t stage_bytes, int max_rows) {
-  extern __shared__ __align__(128) uint8_t smem[];
+__device__ void consume_block_row(const GradRowsArgs& a, const Smem& sm, const StageCfg& c, int64_t rb) {
   using V = Vec<T, VEC>;
   constexpr int E = NCH * VEC;
-  const SmemMap sm = carve(smem, S, max_rows, SR, true);
-  const WorkItem it = a.items[blockIdx.x];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tid = threadIdx.x;
-  const int64_t rb = a.ld * (int64_t)sizeof(T);
-  const int nst = (int)((it.rows + SR - 1) / SR);
-  __shared__ int cta_err;
-
-  if (threadIdx.x == 0) {
-    cta_err = 0;
-    for (int s = 0; s < S; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kNW);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+  ConsumerSync bar{sm.sync, 0u, a.status};
+  if (a.pdl) grid_dep_wait();
+  float wr[E], acc[E];
+#pragma unroll
+  for (int j = 0; j < NCH; ++j)
+#pragma unroll
+    for (int v = 0; v < VEC; ++v) {
+      wr[j * VEC + v] = a.w[(j * kNT + tid) * VEC + v];
+      acc[j * VEC + v] = 0.f;
     }
-    fence_mbar_init();
-  }
-  __syncthreads();
-
-  if (warp == kNW) {
-    if (lane == 0)
-      produce(sm, reinterpret_cast<const uint8_t*>(a.X) + it.row0 * rb, it.rows, rb, SR, S, stage_bytes,
-              a.status);
-  } else {
-    for (int64_t r = tid; r < it.rows; r += kNT) sm.ylab[r] = a.y[it.row0 + r];
-    float wr[E], acc[E];
+  uint32_t ends = 0;
+  bool ok = true;
+  for (int i = 0; ok; ++i) {
+    const int s = i % c.S;
+    if (!__all_sync(0xffffffffu, mbar_wait(&sm.full[s], (i / c.S) & 1, a.status))) { ok = false; break; }
+    const StageHdr h = sm.hdr[s];
+    if (h.item < 0) break;
+    const uint8_t* st = sm.stages + (size_t)s * c.stage_bytes;
+    const float* lab = sm.lab + (size_t)s * c.LS + h.lab_off;
+    float* xd = sm.xdot + (size_t)(i & 1) * c.SR * kNW;
+    for (int rr = 0; rr < h.rows; ++rr) {
+      const typename V::raw* row = reinterpret_cast<const typename V::raw*>(st + rr * rb);
+      float dot = 0.f;
 #pragma unroll
-    for (int j = 0; j < NCH; ++j)
+      for (int j = 0; j < NCH; ++j) {
+        float x[VEC];
+        V::widen(row[j * kNT + tid], x);
 #pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        wr[j * VEC + v] = a.w[(j * kNT + tid) * VEC + v];
-        acc[j * VEC + v] = 0.f;
+        for (int v = 0; v < VEC; ++v) dot = fmaf(x[v], wr[j * VEC + v], dot);
       }
-    named_bar_sync(1, kNT);
-    bool ok = true;
-    for (int i = 0; i < nst; ++i) {
-      const int s = i % S;
-      // Every consumer warp runs all nst iterations and reaches every named
-      // barrier; once a wait has timed out the warp only skips its waits and
-      // arithmetic, and the CTA's result is dropped at the end.
-      if (ok && !__all_sync(0xffffffffu, mbar_wait(&sm.full[s], (i / S) & 1, a.status))) {
-        ok = false;
-        if (lane == 0) atomicExch(&cta_err, 1);
-      }
-      const int rows_i = (int)(it.rows - (int64_t)i * SR < SR ? it.rows - (int64_t)i * SR : SR);
-      const uint8_t* st = sm.stages + (size_t)s * stage_bytes;
-      float* xd = sm.xdot + (size_t)(i & 1) * SR * kNW;
-      for (int rr = 0; rr < rows_i; ++rr) {
-        float dot = 0.f;
-        if (ok) {
-          const typename V::raw* row = reinterpret_cast<const typename V::raw*>(st + rr * rb);
-#pragma unroll
-          for (int j = 0; j < NCH; ++j) {
-            float x[VEC];
-            V::widen(row[j * kNT + tid], x);
-#pragma unroll
-            for (int v = 0; v < VEC; ++v) dot = fmaf(x[v], wr[j * VEC + v], dot);
-          }
-        }
-        dot = warp_sum(dot);
-        if (lane == 0) xd[rr * kNW + warp] = dot;
-      }
-      named_bar_sync(1, kNT);
-      if (ok) {
-        for (int rr = 0; rr < rows_i; ++rr) {
-          float dot = 0.f;
-#pragma unroll
-          for (int w8 = 0; w8 < kNW; ++w8) dot += xd[rr * kNW + w8];
-          const float r = residual(a.loss, dot, sm.ylab[(int64_t)i * SR + rr]);
-          const typename V::raw* row = reinterpret_cast<const typename V::raw*>(st + rr * rb);
-#pragma unroll
-          for (int j = 0; j < NCH; ++j) {
-            float x[VEC];
-            V::widen(row[j * kNT + tid], x);
-#pragma unroll
-            for (int v = 0; v < VEC; ++v) acc[j * VEC + v] = fmaf(r, x[v], acc[j * VEC + v]);
-          }
-        }
-      }
-      __syncwarp();
-      if (lane == 0 && ok) mbar_arrive(&sm.empty[s]);
+      dot = warp_sum(dot);
+      if (lane == 0) xd[rr * kNW + warp] = dot;
     }
-    named_bar_sync(1, kNT);
-    if (!cta_err) {
-      float* out = a.partials + (size_t)blockIdx.x * a.ld;
+    // the exchange buffer alternates by stage parity; the barrier of stage
+    // i + 1 separates this stage's reads from stage i + 2's writes
+    if (!bar()) { ok = false; break; }
+    for (int rr = 0; rr < h.rows; ++rr) {
+      float dot = 0.f;
+#pragma unroll
+      for (int w8 = 0; w8 < kNW; ++w8) dot += xd[rr * kNW + w8];
+      const float r = residual(a.loss, dot, lab[rr]);
+      const typename V::raw* row = reinterpret_cast<const typename V::raw*>(st + rr * rb);
+#pragma unroll
+      for (int j = 0; j < NCH; ++j) {
+        float x[VEC];
+        V::widen(row[j * kNT + tid], x);
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) acc[j * VEC + v] = fmaf(r, x[v], acc[j * VEC + v]);
+      }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&sm.empty[s]);
+    if (h.last) {
+      if (!handover_begin(a, sm, ends, bar, ok)) break;
+      // each thread owns its columns: write them straight to the item's partial
+      float* out = a.partials + (size_t)h.item * a.ld;
 #pragma unroll
       for (int j = 0; j < NCH; ++j)
 #pragma unroll
-        for (int v = 0; v < VEC; ++v) out[(j * kNT + tid) * VEC + v] = acc[j * VEC + v];
+        for (int v = 0; v < VEC; ++v) {
+          out[(j * kNT + tid) * VEC + v] = acc[j * VEC + v];
+          acc[j * VEC + v] = 0.f;
+        }
+      handover_end(sm, h.item, h.e, ends);
     }
+  }
+  consumers_finish(a, sm, ends, bar, ok);
+  if (!ok) atomicOr(a.status, kErrWaitTimeout);
+}
+
+template <typename T, int VEC, int NCH, bool BLOCK>
+__global__ void __launch_bounds__(kThreads, 1) grad_rows_kernel(GradRowsArgs a, StageCfg c) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  const Smem sm = carve(smem, c, BLOCK);
+  const int64_t rb = a.ld * (int64_t)sizeof(T);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < c.S; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kNW);
+    }
+    mbar_init(sm.sync, kNW);
+    mbar_init(sm.red_full, kNW);
+    mbar_init(sm.red_free, 1);
+    sm.ho->item = -1;
+    sm.ho->e = -1;
+    sm.ho->commit = -1;
+    sm.ho->decode = 0;
+    fence_mbar_init();
+    grid_dep_launch();
+  }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5;
+  if (warp == kTailWarp) {
+    tail_warp(a, sm, !BLOCK);
+  } else if (threadIdx.x >= kNT) {
+    if (threadIdx.x == kProducer) produce(a, sm, c, rb);
+  } else if (BLOCK) {
+    consume_block_row<T, VEC, NCH>(a, sm, c, rb);
+  } else {
+    consume_warp_row<T, VEC, NCH>(a, sm, c, rb);
   }
   __syncthreads();
 }
@@ -300,7 +509,7 @@ int grad_rows_variant(int dtype, int64_t d, int64_t* ld_out) {
   return -1;
 }
 
-static StageCfg stage_cfg(int variant, int64_t ld, int max_rows) {
+static StageCfg stage_cfg(int variant, int64_t ld, bool need_decode_scratch) {
   const bool block = variant >= 64;
   const int esz = (variant & 32) ? 2 : 4;
   const int64_t rb = ld * esz;
@@ -314,65 +523,76 @@ static StageCfg stage_cfg(int variant, int64_t ld, int max_rows) {
     c.SR = sr < 1 ? 1 : (sr > 8 ? 8 : sr);
   }
   c.stage_bytes = (uint32_t)(c.SR * rb);
-  size_t fixed = 128 + (((size_t)max_rows * 4 + 127) & ~size_t(127));
-  if (block) fixed += ((size_t)2 * c.SR * kNW * 4 + 127) & ~size_t(127);
-  const size_t budget = 200 * 1024;
-  int S = (int)((budget - fixed) / c.stage_bytes);
-  c.S = S > 8 ? 8 : S;
-  c.smem = fixed + (size_t)c.S * c.stage_bytes;
-  // the warp-row epilogue reuses the stages for kNW * ld fp32 values
+  c.LS = ((c.SR + 3 + 3) / 4) * 4;   // labels of SR rows read from a 4-row-aligned start
+  const size_t red = block ? 0 : (size_t)kNW * ld * sizeof(float);
+  c.red_bytes = red;
+  c.plan_bytes = need_decode_scratch ? sizeof(DecodePlan) : 0;
+  const size_t budget = 220 * 1024;
+  int S = 8;
+  while (S > 2 && fixed_bytes(S, c.LS, red, c.SR, block, c.plan_bytes) + (size_t)S * c.stage_bytes > budget) --S;
+  c.S = S;
+  c.smem = fixed_bytes(S, c.LS, red, c.SR, block, c.plan_bytes) + (size_t)S * c.stage_bytes;
   return c;
 }
 
 int grad_rows_stage_rows(int variant, int64_t ld, int dtype) {
   (void)dtype;
-  return stage_cfg(variant, ld, 1).SR;
+  return stage_cfg(variant, ld, false).SR;
 }
 
 template <typename K>
-static cudaError_t launch_k(K kern, const GradRowsArgs& a, const StageCfg& c, int max_rows, cudaStream_t st) {
+static cudaError_t launch_k(K kern, const GradRowsArgs& a, const StageCfg& c, int grid, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)c.smem);
   if (e != cudaSuccess) return e;
-  kern<<<a.nitems, kThreads, c.smem, st>>>(a, c.SR, c.S, c.stage_bytes, max_rows);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = c.smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = a.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kern, a, c);
 }
 
-#define PGC_WR(T, VEC, NCH) grad_rows_warp<T, VEC, NCH>
-#define PGC_BR(T, VEC, NCH) grad_rows_block<T, VEC, NCH>
+#define PGC_WR(T, VEC, NCH) grad_rows_kernel<T, VEC, NCH, false>
+#define PGC_BR(T, VEC, NCH) grad_rows_kernel<T, VEC, NCH, true>
 
 cudaError_t launch_grad_rows(const GradRowsArgs& a, int variant, cudaStream_t st) {
   if (a.nitems <= 0) return cudaSuccess;
-  // the largest item decides the label buffer; the host caps items
-  const int max_rows = a.max_item_rows;
-  if (max_rows < 1 || max_rows > kMaxItemRows) return cudaErrorInvalidValue;
-  const StageCfg c = stage_cfg(variant, a.ld, max_rows);
-  if (c.S < 2) return cudaErrorInvalidValue;
+  const StageCfg c = stage_cfg(variant, a.ld, a.tail == 2);
+  if (c.smem > 227 * 1024) return cudaErrorInvalidValue;
+  // persistent grid when items are taken dynamically, else one CTA per item
+  const int grid = a.work_ctr ? (a.grid < a.nitems ? a.grid : a.nitems) : a.nitems;
+  if (grid < 1) return cudaErrorInvalidValue;
   switch (variant) {
     // warp-row fp32: VEC 1,2,4 (NCH 1) and VEC 4 with NCH 2..8
-    case 0 * 8 + 0: return launch_k(PGC_WR(float, 1, 1), a, c, max_rows, st);
-    case 1 * 8 + 0: return launch_k(PGC_WR(float, 2, 1), a, c, max_rows, st);
-    case 2 * 8 + 0: return launch_k(PGC_WR(float, 4, 1), a, c, max_rows, st);
-    case 2 * 8 + 1: return launch_k(PGC_WR(float, 4, 2), a, c, max_rows, st);
-    case 2 * 8 + 2: return launch_k(PGC_WR(float, 4, 4), a, c, max_rows, st);
-    case 2 * 8 + 3: return launch_k(PGC_WR(float, 4, 8), a, c, max_rows, st);
+    case 0 * 8 + 0: return launch_k(PGC_WR(float, 1, 1), a, c, grid, st);
+    case 1 * 8 + 0: return launch_k(PGC_WR(float, 2, 1), a, c, grid, st);
+    case 2 * 8 + 0: return launch_k(PGC_WR(float, 4, 1), a, c, grid, st);
+    case 2 * 8 + 1: return launch_k(PGC_WR(float, 4, 2), a, c, grid, st);
+    case 2 * 8 + 2: return launch_k(PGC_WR(float, 4, 4), a, c, grid, st);
+    case 2 * 8 + 3: return launch_k(PGC_WR(float, 4, 8), a, c, grid, st);
     // warp-row bf16: VEC 2,4,8 (NCH 1) and VEC 8 with NCH 2..8
-    case 32 + 1 * 8 + 0: return launch_k(PGC_WR(uint16_t, 2, 1), a, c, max_rows, st);
-    case 32 + 2 * 8 + 0: return launch_k(PGC_WR(uint16_t, 4, 1), a, c, max_rows, st);
-    case 32 + 3 * 8 + 0: return launch_k(PGC_WR(uint16_t, 8, 1), a, c, max_rows, st);
-    case 32 + 3 * 8 + 1: return launch_k(PGC_WR(uint16_t, 8, 2), a, c, max_rows, st);
-    case 32 + 3 * 8 + 2: return launch_k(PGC_WR(uint16_t, 8, 4), a, c, max_rows, st);
-    case 32 + 3 * 8 + 3: return launch_k(PGC_WR(uint16_t, 8, 8), a, c, max_rows, st);
+    case 32 + 1 * 8 + 0: return launch_k(PGC_WR(uint16_t, 2, 1), a, c, grid, st);
+    case 32 + 2 * 8 + 0: return launch_k(PGC_WR(uint16_t, 4, 1), a, c, grid, st);
+    case 32 + 3 * 8 + 0: return launch_k(PGC_WR(uint16_t, 8, 1), a, c, grid, st);
+    case 32 + 3 * 8 + 1: return launch_k(PGC_WR(uint16_t, 8, 2), a, c, grid, st);
+    case 32 + 3 * 8 + 2: return launch_k(PGC_WR(uint16_t, 8, 4), a, c, grid, st);
+    case 32 + 3 * 8 + 3: return launch_k(PGC_WR(uint16_t, 8, 8), a, c, grid, st);
     // block-row fp32 (VEC 4) and bf16 (VEC 8), NCH 1..16
-    case 64 + 2 * 8 + 0: return launch_k(PGC_BR(float, 4, 1), a, c, max_rows, st);
-    case 64 + 2 * 8 + 1: return launch_k(PGC_BR(float, 4, 2), a, c, max_rows, st);
-    case 64 + 2 * 8 + 2: return launch_k(PGC_BR(float, 4, 4), a, c, max_rows, st);
-    case 64 + 2 * 8 + 3: return launch_k(PGC_BR(float, 4, 8), a, c, max_rows, st);
-    case 64 + 2 * 8 + 4: return launch_k(PGC_BR(float, 4, 16), a, c, max_rows, st);
-    case 64 + 32 + 3 * 8 + 0: return launch_k(PGC_BR(uint16_t, 8, 1), a, c, max_rows, st);
-    case 64 + 32 + 3 * 8 + 1: return launch_k(PGC_BR(uint16_t, 8, 2), a, c, max_rows, st);
-    case 64 + 32 + 3 * 8 + 2: return launch_k(PGC_BR(uint16_t, 8, 4), a, c, max_rows, st);
-    case 64 + 32 + 3 * 8 + 3: return launch_k(PGC_BR(uint16_t, 8, 8), a, c, max_rows, st);
-    case 64 + 32 + 3 * 8 + 4: return launch_k(PGC_BR(uint16_t, 8, 16), a, c, max_rows, st);
+    case 64 + 2 * 8 + 0: return launch_k(PGC_BR(float, 4, 1), a, c, grid, st);
+    case 64 + 2 * 8 + 1: return launch_k(PGC_BR(float, 4, 2), a, c, grid, st);
+    case 64 + 2 * 8 + 2: return launch_k(PGC_BR(float, 4, 4), a, c, grid, st);
+    case 64 + 2 * 8 + 3: return launch_k(PGC_BR(float, 4, 8), a, c, grid, st);
+    case 64 + 2 * 8 + 4: return launch_k(PGC_BR(float, 4, 16), a, c, grid, st);
+    case 64 + 32 + 3 * 8 + 0: return launch_k(PGC_BR(uint16_t, 8, 1), a, c, grid, st);
+    case 64 + 32 + 3 * 8 + 1: return launch_k(PGC_BR(uint16_t, 8, 2), a, c, grid, st);
+    case 64 + 32 + 3 * 8 + 2: return launch_k(PGC_BR(uint16_t, 8, 4), a, c, grid, st);
+    case 64 + 32 + 3 * 8 + 3: return launch_k(PGC_BR(uint16_t, 8, 8), a, c, grid, st);
+    case 64 + 32 + 3 * 8 + 4: return launch_k(PGC_BR(uint16_t, 8, 16), a, c, grid, st);
     default: return cudaErrorInvalidValue;
   }
 }

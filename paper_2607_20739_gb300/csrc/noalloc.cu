@@ -29,13 +29,12 @@
 #include <cstring>
 #include <mutex>
 
-#include "../../include/pgc.h"
+#include "pgc.h"
 #include "pgc_internal.h"
 
 namespace {
 
 constexpr size_t kScratchBytes = size_t(16) << 20;   // 16 MiB
-constexpr int kMaxItemRowsNA = 8192;                 // rows of one CTA's work item
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
@@ -106,20 +105,26 @@ extern "C" int pgc_gradient_noalloc(int32_t loss, int32_t dtype, int64_t m, int6
       cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return PGC_ECUDA;
 
-  // one work item per SM, at least one stage of rows each, at most 8192 rows
+  // one work item (one CTA) per SM, at least one stage of rows each
   const int64_t sr = pgc::grad_rows_stage_rows(variant, ld, dtype);
   int64_t G = std::min<int64_t>(sms, (m + sr - 1) / sr);
-  G = std::max<int64_t>(G, (m + kMaxItemRowsNA - 1) / kMaxItemRowsNA);
   G = std::max<int64_t>(G, 1);
-  const size_t off_partials = align256(kOffItems + (size_t)G * sizeof(pgc::WorkItem));
+  // the gradient kernel copies labels per stage from a 16-byte aligned start
+  // and may read 12 bytes past the last one, so it reads a padded copy here
+  const size_t off_labels = align256(kOffItems + (size_t)G * sizeof(pgc::WorkItem));
+  const size_t off_partials = align256(off_labels + (size_t)m * sizeof(float) + 16);
   if (off_partials + (size_t)G * (size_t)ld * sizeof(float) > kScratchBytes) return PGC_ESCRATCH;
 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   noalloc_fill_tables<<<(unsigned)((G + 255) / 256), 256, 0, st>>>(scratch, (int)G, m);
   if (cudaGetLastError() != cudaSuccess) return PGC_ECUDA;
+  if (cudaMemcpyAsync(scratch + off_labels, y, (size_t)m * sizeof(float), cudaMemcpyDeviceToDevice, st) !=
+      cudaSuccess)
+    return PGC_ECUDA;
 
   pgc::GradRowsArgs g;
-  g.loss = loss; g.dtype = dtype; g.d = d; g.ld = ld; g.X = X; g.y = y; g.w = w;
+  g.loss = loss; g.dtype = dtype; g.d = d; g.ld = ld; g.X = X;
+  g.y = reinterpret_cast<const float*>(scratch + off_labels); g.w = w;
   g.items = reinterpret_cast<const pgc::WorkItem*>(scratch + kOffItems);
   g.nitems = (int)G;
   int64_t max_rows = 0;

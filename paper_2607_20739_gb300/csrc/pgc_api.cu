@@ -22,14 +22,12 @@
 #include <new>
 #include <vector>
 
-#include "../../include/pgc.h"
+#include "pgc.h"
 #include "pgc_internal.h"
 
 using namespace pgc;
 
 namespace {
-
-constexpr int kItemMaxRows = 8192;
 
 struct Phase {
   int slot = -1;                        // o, or -1 for the warm-up
@@ -99,6 +97,10 @@ struct pgc_ctx {
   double* loss_blocks = nullptr;
   double* loss_out = nullptr;
   int64_t* loss_desc = nullptr;
+  int* counters = nullptr;   // [n + 3]: per-partition arrivals, committed partitions,
+                             // work-item counter, finished producers (zero between steps)
+  bool pdl = true;           // chain the step's kernels with programmatic dependent launch
+  int tail_mode = 0;         // fused tail of the gradient kernel (see GradRowsArgs)
   int64_t loss_chunk = 0;
   int loss_nblocks = 256;
   void* tables = nullptr;
@@ -179,18 +181,19 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
   }
   ph.z_total = R;
   if (ctx->loss != PGC_SOFTMAX) {
-    // split rows into about sm_count * waves items of similar size
-    const double bytes = (double)R * ctx->ld * ctx->esize;
-    const int waves = bytes > 1e9 ? 3 : 1;
-    const int64_t G = (int64_t)ctx->sm_count * waves;
+    // work items per SM (default 1: one balanced static item per CTA; more are
+    // taken dynamically by the persistent grid);
+    // an item holds at least one stage of rows.  PGC_ITEMS_PER_SM overrides.
+    int per_sm = 1;
+    if (const char* env = std::getenv("PGC_ITEMS_PER_SM")) per_sm = std::max(1, std::atoi(env));
+    const int64_t G = (int64_t)ctx->sm_count * per_sm;
     const int64_t min_rows = grad_rows_stage_rows(ctx->variant, ctx->ld, ctx->dtype);
     ph.e_item0.push_back(0);
     for (int e = 0; e < nE; ++e) {
       const int64_t m = ph.e_rows[e];
       int64_t q = (int64_t)std::llround((double)G * (double)m / (double)R);
       q = std::max<int64_t>(q, 1);
-      q = std::min<int64_t>(q, std::max<int64_t>(1, (m + min_rows - 1) / min_rows));
-      q = std::max<int64_t>(q, (m + kItemMaxRows - 1) / kItemMaxRows);
+      q = std::min<int64_t>(q, std::max<int64_t>(1, m / min_rows));
       for (int64_t i = 0; i < q; ++i) {
         const int64_t a = m * i / q, b = m * (i + 1) / q;
         WorkItem it;
@@ -232,7 +235,7 @@ void free_all(pgc_ctx* ctx) {
   for (cudaEvent_t ev : ctx->ev_pool) cudaEventDestroy(ev);
   ctx->ev_pool.clear();
   void* ptrs[] = {ctx->X, ctx->y, ctx->w, ctx->wb, ctx->store, ctx->U, ctx->gout, ctx->partials, ctx->Z,
-                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->loss_desc, ctx->tables};
+                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->tables, ctx->counters};
   for (void* p : ptrs)
     if (p) cudaFree(p);
 }
@@ -319,6 +322,17 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   }
   ctx->P = ctx->K * ctx->ld;
   ctx->Kpad = (int64_t)align_up((size_t)K, 4);
+  {
+    const char* env = std::getenv("PGC_NO_PDL");
+    ctx->pdl = !(env && env[0] == '1');
+  }
+  if (loss != PGC_SOFTMAX) {
+    // fuse the decode into the gradient kernel when one CTA can read what it
+    // needs quickly: the refreshed slot of every store, the other slot
+    // totals and the stragglers' stores, about (owners + c + s c) P floats
+    const double dec_bytes = (double)(ctx->owners + ctx->c + (double)s * ctx->c) * ctx->P * 4.0;
+    ctx->tail_mode = dec_bytes <= 512.0 * 1024.0 ? 2 : 1;
+  }
 
   cudaError_t e = cudaGetDevice(&ctx->device);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sm_count, cudaDevAttrMultiProcessorCount, ctx->device);
@@ -374,7 +388,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
 
   const size_t Pb = (size_t)ctx->P * sizeof(float);
   PGC_ALLOC(ctx->X, (size_t)ctx->total_rows * ctx->ld * ctx->esize);
-  PGC_ALLOC(ctx->y, (size_t)ctx->total_rows * 4);
+  PGC_ALLOC(ctx->y, (size_t)ctx->total_rows * 4 + 64);   // per-stage label copies overrun by <= 12 B
   PGC_ALLOC(ctx->w, Pb);
   if (dtype == PGC_BF16) PGC_ALLOC(ctx->wb, (size_t)ctx->P * 2);
   PGC_ALLOC(ctx->store, (size_t)ctx->owners * ctx->c * Pb);
@@ -388,6 +402,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   PGC_ALLOC(ctx->loss_blocks, (size_t)ctx->loss_nblocks * sizeof(double));
   PGC_ALLOC(ctx->loss_out, sizeof(double));
   PGC_ALLOC(ctx->tables, tab.size());
+  PGC_ALLOC(ctx->counters, (size_t)(n + 3) * sizeof(int));
 
   cudaStream_t st = ctx->stream;
   e = cudaMemcpyAsync(ctx->tables, tab.data(), tab.size(), cudaMemcpyHostToDevice, st);
@@ -398,6 +413,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->gout, 0, Pb, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->coeff, 0, (size_t)n * sizeof(float), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->status, 0, sizeof(int), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ctx->counters, 0, (size_t)(n + 3) * sizeof(int), st);
   if (e == cudaSuccess && w0)
     e = cudaMemcpy2DAsync(ctx->w, ctx->ld * sizeof(float), w0, d * sizeof(float), d * sizeof(float), K,
                           cudaMemcpyHostToDevice, st);
@@ -471,16 +487,33 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
   cudaStream_t st = ctx->stream;
 
   PGC_CK(ctx, record_event(ctx));
-  int64_t nl[PGC_NKGROUPS] = {0, 1, 1};
-  // K1 / softmax gradient -> partials
+  int64_t nl[PGC_NKGROUPS] = {0, 0, 0};
+  DecodeArgs dc;
+  dc.scheme = ctx->scheme; dc.n = n; dc.s = ctx->s; dc.c = c; dc.slot = ph.slot; dc.owners = ctx->owners;
+  dc.mask = bits; dc.P = ctx->P; dc.store = ctx->store; dc.U = ctx->U; dc.w = ctx->w; dc.wb = ctx->wb;
+  dc.gout = ctx->gout; dc.lr = ctx->lr; dc.coeff_out = ctx->coeff; dc.status = ctx->status;
+  // device outputs with the unpadded layout (ld == d) and 16-byte alignment are
+  // written by the decode itself, so no copy sits between consecutive steps
+  const bool direct = outputs_on_device && ctx->ld == ctx->d &&
+                      (reinterpret_cast<uintptr_t>(grad_out) % 16 == 0) && (reinterpret_cast<uintptr_t>(w_out) % 16 == 0);
+  if (direct) { dc.g_user = grad_out; dc.w_user = w_out; }
+  bool need_commit = true, need_decode = true;
   if (ctx->loss != PGC_SOFTMAX) {
-    nl[PGC_KGRAD] = ph.items.empty() ? 0 : 1;
+    // K1 with its fused tail: commit (and, for small P, decode) in the same launch
     GradRowsArgs g;
     g.loss = ctx->loss; g.dtype = ctx->dtype; g.d = ctx->d; g.ld = ctx->ld;
     g.X = ctx->X; g.y = static_cast<const float*>(ctx->y); g.w = ctx->w;
     g.items = ph.d_items; g.nitems = (int)ph.items.size(); g.max_item_rows = ph.max_item_rows;
     g.partials = ctx->partials; g.status = ctx->status;
+    g.tail = ctx->tail_mode; g.pdl = ctx->pdl;
+    g.cnt_e = ctx->counters; g.cnt_all = ctx->counters + n;
+    g.work_ctr = ctx->counters + n + 1; g.prod_done = ctx->counters + n + 2; g.grid = ctx->sm_count;
+    g.e_item0 = ph.d_e_item0; g.e_scale = ph.d_e_scale; g.e_dest = ph.d_e_dest; g.ndest = ph.ndest;
+    g.nE = (int)ph.parts.size(); g.store = ctx->store; g.dec = dc;
+    nl[PGC_KGRAD] = 1;
     PGC_CK(ctx, launch_grad_rows(g, ctx->variant, st));
+    need_commit = false;
+    need_decode = ctx->tail_mode < 2;
   } else {
     SoftmaxCCArgs a;
     a.dtype = ctx->dtype; a.ld = ctx->ld; a.K = ctx->K; a.X = ctx->X; a.y = static_cast<const int32_t*>(ctx->y);
@@ -491,26 +524,28 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     PGC_CK(ctx, launch_softmax_cc(a, st));
   }
   PGC_CK(ctx, record_event(ctx));
-  // K4 commit into the stores
-  CommitArgs cm;
-  cm.partials = ctx->partials; cm.P = ctx->P; cm.e_item0 = ph.d_e_item0; cm.e_scale = ph.d_e_scale;
-  cm.e_dest = ph.d_e_dest; cm.ndest = ph.ndest; cm.nE = (int)ph.parts.size(); cm.store = ctx->store;
-  PGC_CK(ctx, launch_commit(cm, st));
+  if (need_commit) {
+    // K4 commit into the stores
+    CommitArgs cm;
+    cm.partials = ctx->partials; cm.P = ctx->P; cm.e_item0 = ph.d_e_item0; cm.e_scale = ph.d_e_scale;
+    cm.e_dest = ph.d_e_dest; cm.ndest = ph.ndest; cm.nE = (int)ph.parts.size(); cm.store = ctx->store;
+    nl[PGC_KCOMMIT] = 1;
+    PGC_CK(ctx, launch_commit(cm, st, ctx->pdl));
+  }
   PGC_CK(ctx, record_event(ctx));
-  // K5+K6 decode + SGD
-  DecodeArgs dc;
-  dc.scheme = ctx->scheme; dc.n = n; dc.s = ctx->s; dc.c = c; dc.slot = ph.slot; dc.owners = ctx->owners;
-  dc.mask = bits; dc.P = ctx->P; dc.store = ctx->store; dc.U = ctx->U; dc.w = ctx->w; dc.wb = ctx->wb;
-  dc.gout = ctx->gout; dc.lr = ctx->lr; dc.coeff_out = ctx->coeff; dc.status = ctx->status;
-  PGC_CK(ctx, launch_decode(dc, st));
+  if (need_decode) {
+    // K5+K6 decode + SGD
+    nl[PGC_KDECODE] = 1;
+    PGC_CK(ctx, launch_decode(dc, st, ctx->pdl, ctx->sm_count));
+  }
   PGC_CK(ctx, record_event(ctx));
   if (ctx->timing) {
     for (int k = 0; k < PGC_NKGROUPS; ++k) ctx->launches[k] += nl[k];
     ++ctx->timed_steps;
   }
 
-  if (grad_out) { int rc = copy_out(ctx, grad_out, ctx->gout, outputs_on_device); if (rc) return rc; }
-  if (w_out) { int rc = copy_out(ctx, w_out, ctx->w, outputs_on_device); if (rc) return rc; }
+  if (grad_out && !direct) { int rc = copy_out(ctx, grad_out, ctx->gout, outputs_on_device); if (rc) return rc; }
+  if (w_out && !direct) { int rc = copy_out(ctx, w_out, ctx->w, outputs_on_device); if (rc) return rc; }
   if (!outputs_on_device && (grad_out || w_out)) {
     const int rc = read_status(ctx);
     if (rc) return rc;

@@ -24,6 +24,28 @@ struct WorkItem {
   int64_t rows;     // number of rows (>= 1)
 };
 
+// ---- K5 + K6: decode coefficients from the mask, decode, SGD --------------
+constexpr int kMaxWorkers = 1024;
+struct MaskBits {
+  uint32_t w[kMaxWorkers / 32];
+};
+struct DecodeArgs {
+  int scheme, n, s, c;
+  int slot;                 // o_t refreshed this step, or -1: all slots (warm-up)
+  int owners;               // stores: n (CR) or n / c (FR groups)
+  MaskBits mask;            // bit i = 1: worker i straggles
+  int64_t P;                // floats per gradient (multiple of 4)
+  float* store;             // [owners * c][P]
+  float* U;                 // [c][P] slot totals
+  float* w;                 // [P] parameters, updated in place
+  uint16_t* wb;             // [P] bf16 copy of w, or nullptr
+  float* gout;              // [P] decoded gradient
+  float lr;
+  float* coeff_out;         // [n] per-worker coefficient a_i (written once per step)
+  int* status;
+  float* g_user = nullptr;  // optional extra destinations of ghat and beta, same
+  float* w_user = nullptr;  // unpadded layout (used when ld == d)
+};
 // ---- K1: streaming gradient of logistic / least-squares partitions -------
 // For every work item: partial[item][0:ld] = sum over its rows x of
 // residual(x) * x, residual = sigmoid(x.w) - y (logistic) or x.w - y (lsq).
@@ -36,9 +58,32 @@ struct GradRowsArgs {
   const float* w;           // parameters [ld] (padding is zero)
   const WorkItem* items;    // device [nitems]
   int nitems;
-  int max_item_rows;        // rows of the largest item (<= 8192)
+  int max_item_rows;        // rows of the largest item
   float* partials;          // [nitems][ld]
+  // Labels are copied per stage from a 16-byte aligned start, so up to 12
+  // bytes past the last label are read: y must be padded by 16 bytes.
+  // Dynamic scheduling: with work_ctr set, `grid` persistent CTAs take items
+  // blockIdx.x, then gridDim.x + atomicAdd(work_ctr, 1); the last producer
+  // resets work_ctr and prod_done.  Without it, one CTA per item.
+  int* work_ctr = nullptr;
+  int* prod_done = nullptr;
+  int grid = 0;
   int* status;              // device status word (error bits)
+  // Fused tail.  tail = 0: partial sums only.  1: the last CTA of each
+  // partition also commits it (ordered sum of its partials, scaled, into its
+  // destination stores).  2: additionally the CTA committing the last
+  // partition derives the decode coefficients, decodes and updates w (dec).
+  int tail = 0;
+  bool pdl = false;         // programmatic dependent: consumers wait before reading w
+  int* cnt_e = nullptr;     // [nE] arrivals per partition, zero between steps
+  int* cnt_all = nullptr;   // committed partitions, zero between steps
+  const int32_t* e_item0 = nullptr;
+  const float* e_scale = nullptr;
+  const int32_t* e_dest = nullptr;
+  int ndest = 1;
+  int nE = 0;
+  float* store = nullptr;   // [owners * c][ld]
+  DecodeArgs dec;           // used when tail == 2
 };
 int grad_rows_variant(int dtype, int64_t d, int64_t* ld_out);  // chooses ld, returns variant id
 int grad_rows_stage_rows(int variant, int64_t ld, int dtype);
@@ -58,29 +103,9 @@ struct CommitArgs {
   int nE;
   float* store;             // [owners * c][P]
 };
-cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st);
+cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl = false);
 
-// ---- K5 + K6: decode coefficients from the mask, decode, SGD --------------
-constexpr int kMaxWorkers = 1024;
-struct MaskBits {
-  uint32_t w[kMaxWorkers / 32];
-};
-struct DecodeArgs {
-  int scheme, n, s, c;
-  int slot;                 // o_t refreshed this step, or -1: all slots (warm-up)
-  int owners;               // stores: n (CR) or n / c (FR groups)
-  MaskBits mask;            // bit i = 1: worker i straggles
-  int64_t P;                // floats per gradient (multiple of 4)
-  float* store;             // [owners * c][P]
-  float* U;                 // [c][P] slot totals
-  float* w;                 // [P] parameters, updated in place
-  uint16_t* wb;             // [P] bf16 copy of w, or nullptr
-  float* gout;              // [P] decoded gradient
-  float lr;
-  float* coeff_out;         // [n] per-worker coefficient a_i (written by CTA 0)
-  int* status;
-};
-cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st, bool pdl, int sm_count);
 
 // ---- generic softmax gradient on CUDA cores --------------------------------
 // logits Z[r][k] = sum_j W[k][j] x_r[j] for the rows of each evaluated

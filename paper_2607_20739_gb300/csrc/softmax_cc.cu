@@ -6,7 +6,7 @@
 // Also provides the tiled logits pass used by the full-loss kernel.
 #include "dev_common.cuh"
 #include "pgc_internal.h"
-#include "../../include/pgc.h"
+#include "pgc.h"
 
 namespace pgc {
 
