@@ -52,7 +52,22 @@ def parse_args(argv=None):
     ap.add_argument("--seed", type=int, default=1)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle sample")
+    ap.add_argument("--override", action="append", default=[],
+                    help="KEY=VALUE change of the workload (n, s, m, d, K) for profiling smaller cases")
     return ap.parse_args(argv)
+
+
+def workload_from_args(args) -> W.Workload:
+    w = W.WORKLOADS[args.workload]
+    kw = {}
+    for o in args.override:
+        k, v = o.split("=", 1)
+        if k not in ("n", "s", "m", "d", "K"):
+            raise SystemExit(f"cannot override {k}")
+        kw[k] = int(v)
+    if kw:
+        w = w.replace(name=w.name + "+" + ",".join(f"{k}={v}" for k, v in sorted(kw.items())), **kw)
+    return w
 
 
 # ---------------------------------------------------------------------------
@@ -240,7 +255,7 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     from paper_2607_20739_gb300 import binding as B
 
-    w = W.WORKLOADS[args.workload]
+    w = workload_from_args(args)
     K_steps = args.steps or default_steps(w)
     Wu = max(3, args.warmup)
     Xs, ys = W.make_partitions(w, args.seed)
@@ -374,7 +389,7 @@ def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
         return
-    w = W.WORKLOADS[args.workload]
+    w = workload_from_args(args)
     K_steps = args.steps or 3
     Xs, ys = W.make_partitions(w, args.seed)
     masks = W.make_masks(w, K_steps + max(3, args.warmup) + 1, args.seed + 1000)

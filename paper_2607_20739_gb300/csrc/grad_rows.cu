@@ -49,6 +49,8 @@ constexpr int kNT = kNW * 32;          // consumer threads
 constexpr int kThreads = kNT + 64;     // + a producer warp + a tail warp
 constexpr int kProducer = kNT;        // producer thread
 constexpr int kTailWarp = kNW + 1;     // warp index of the tail warp
+constexpr int64_t kPrefetchBytes = 256 * 1024;   // L2 warm-up per CTA at start
+constexpr int64_t kPrefetchChunkRows = 16;
 
 struct StageHdr {
   int item;      // work item, or -1: no more work
@@ -79,6 +81,7 @@ struct Handoff {
   int e;
   int commit;          // set by the tail warp: partition to commit, or -1
   int decode;          // set by the consumers: this CTA decodes
+  unsigned sync_count; // arrivals at the consumer barrier (ConsumerSync)
 };
 
 // Shared memory: [full S | empty S | sync, red_full, red_free, tail_done]
@@ -132,14 +135,26 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const StageCfg& c, bool blo
 }
 
 // A barrier of the 8 consumer warps on an mbarrier (count kNW), bounded.
+// Each warp also counts its arrival on a shared counter; the warp whose
+// arrival is the kNW-th knows every other warp is already through its
+// pre-barrier work and does not wait (waiting on a phase it completed itself
+// was measured to cost microseconds).
 struct ConsumerSync {
   uint64_t* bar;
+  unsigned* count;
   uint32_t phase;
   int* status;
   __device__ __forceinline__ bool operator()() {
     __syncwarp();
-    if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
-    const bool ok = mbar_wait(bar, phase, status);
+    int last = 0;
+    if ((threadIdx.x & 31) == 0) {
+      last = (atomic_add_cta_acq_rel(count, 1u) + 1u) % (unsigned)kNW == 0u;
+      mbar_arrive(bar);
+    }
+    last = __shfl_sync(0xffffffffu, last, 0);
+    __syncwarp();                        // lane 0's acquire covers the whole warp
+    bool ok = true;
+    if (!last) ok = mbar_wait(bar, phase, status);
     phase ^= 1u;
     return __all_sync(0xffffffffu, ok);
   }
@@ -155,6 +170,20 @@ __device__ void produce(const GradRowsArgs& a, const Smem& sm, const StageCfg& c
   int i = 0;                     // stages issued
   bool ok = true, waited = false;
   int item = blockIdx.x;
+  if (item < a.nitems) {
+    // Beyond the S stages it can hold, warm L2 with the next rows of the
+    // first item: a CTA started early by the dependent launch keeps HBM busy
+    // while the previous step finishes, and reads these rows from L2 later.
+    const WorkItem it = a.items[item];
+    const int64_t r0 = it.row0 + (int64_t)c.S * c.SR;
+    int64_t rows = it.rows - (int64_t)c.S * c.SR;
+    const int64_t cap = (int64_t)(kPrefetchBytes / rb);
+    rows = rows < cap ? rows : cap;
+    for (int64_t r = 0; r < rows; r += kPrefetchChunkRows) {
+      const int64_t n = rows - r < kPrefetchChunkRows ? rows - r : kPrefetchChunkRows;
+      prefetch_l2(X + (r0 + r) * rb, (uint32_t)(n * rb));
+    }
+  }
   while (ok && item < a.nitems) {
     const WorkItem it = a.items[item];
     const int nst = (int)((it.rows + c.SR - 1) / c.SR);
@@ -229,11 +258,11 @@ __device__ void tail_warp(const GradRowsArgs& a, const Smem& sm, bool warp_row) 
     if (a.tail) {
       __syncwarp();
       if (lane == 0) {
-        __threadfence();               // the item's partial (written by this warp or by the consumers)
-        const int prev = atomicAdd(&a.cnt_e[e], 1);
+        // release this item's partial (written by this warp, or by the
+        // consumers before red_full) and acquire the other items' partials
+        const int prev = atomic_add_acq_rel(&a.cnt_e[e], 1);
         if (prev == a.e_item0[e + 1] - a.e_item0[e] - 1) {
           a.cnt_e[e] = 0;              // every item of e has arrived: reset for the next step
-          __threadfence();             // acquire the other CTAs' partials before handing e to the consumers
           commit = e;
         }
       }
@@ -256,12 +285,10 @@ __device__ void consumer_commit(const GradRowsArgs& a, const Smem& sm, int e, in
                a.ndest, a.store, tid, kNT);
   if (!bar()) { ok = false; return; }
   if (tid == 0) {
-    __threadfence();                   // release the stores written by the whole CTA
-    const bool all = atomicAdd(a.cnt_all, 1) == a.nE - 1;
-    if (all) {
-      *a.cnt_all = 0;
-      __threadfence();                 // acquire the other committers' stores
-    }
+    // release the stores written by the whole CTA (ordered before this by the
+    // barrier) and acquire the other committers' stores
+    const bool all = atomic_add_acq_rel(a.cnt_all, 1) == a.nE - 1;
+    if (all) *a.cnt_all = 0;
     if (all && a.tail == 2) sm.ho->decode = 1;
   }
 }
@@ -316,7 +343,7 @@ __device__ void consume_warp_row(const GradRowsArgs& a, const Smem& sm, const St
   using V = Vec<T, VEC>;
   constexpr int E = NCH * VEC;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  ConsumerSync bar{sm.sync, 0u, a.status};
+  ConsumerSync bar{sm.sync, &sm.ho->sync_count, 0u, a.status};
   if (a.pdl) grid_dep_wait();                       // w is the previous step's output
   float wr[E], acc[E];
 #pragma unroll
@@ -372,7 +399,7 @@ __device__ void consume_block_row(const GradRowsArgs& a, const Smem& sm, const S
   using V = Vec<T, VEC>;
   constexpr int E = NCH * VEC;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
-  ConsumerSync bar{sm.sync, 0u, a.status};
+  ConsumerSync bar{sm.sync, &sm.ho->sync_count, 0u, a.status};
   if (a.pdl) grid_dep_wait();
   float wr[E], acc[E];
 #pragma unroll
@@ -459,6 +486,7 @@ __global__ void __launch_bounds__(kThreads, 1) grad_rows_kernel(GradRowsArgs a, 
     sm.ho->e = -1;
     sm.ho->commit = -1;
     sm.ho->decode = 0;
+    sm.ho->sync_count = 0;
     fence_mbar_init();
     grid_dep_launch();
   }
@@ -509,7 +537,7 @@ int grad_rows_variant(int dtype, int64_t d, int64_t* ld_out) {
   return -1;
 }
 
-static StageCfg stage_cfg(int variant, int64_t ld, bool need_decode_scratch) {
+static StageCfg stage_cfg(int variant, int64_t ld, int tail) {
   const bool block = variant >= 64;
   const int esz = (variant & 32) ? 2 : 4;
   const int64_t rb = ld * esz;
@@ -526,7 +554,7 @@ static StageCfg stage_cfg(int variant, int64_t ld, bool need_decode_scratch) {
   c.LS = ((c.SR + 3 + 3) / 4) * 4;   // labels of SR rows read from a 4-row-aligned start
   const size_t red = block ? 0 : (size_t)kNW * ld * sizeof(float);
   c.red_bytes = red;
-  c.plan_bytes = need_decode_scratch ? sizeof(DecodePlan) : 0;
+  c.plan_bytes = tail == 2 ? sizeof(DecodePlan) : 0;
   const size_t budget = 220 * 1024;
   int S = 8;
   while (S > 2 && fixed_bytes(S, c.LS, red, c.SR, block, c.plan_bytes) + (size_t)S * c.stage_bytes > budget) --S;
@@ -537,7 +565,7 @@ static StageCfg stage_cfg(int variant, int64_t ld, bool need_decode_scratch) {
 
 int grad_rows_stage_rows(int variant, int64_t ld, int dtype) {
   (void)dtype;
-  return stage_cfg(variant, ld, false).SR;
+  return stage_cfg(variant, ld, 0).SR;
 }
 
 template <typename K>
@@ -562,7 +590,7 @@ static cudaError_t launch_k(K kern, const GradRowsArgs& a, const StageCfg& c, in
 
 cudaError_t launch_grad_rows(const GradRowsArgs& a, int variant, cudaStream_t st) {
   if (a.nitems <= 0) return cudaSuccess;
-  const StageCfg c = stage_cfg(variant, a.ld, a.tail == 2);
+  const StageCfg c = stage_cfg(variant, a.ld, a.tail);
   if (c.smem > 227 * 1024) return cudaErrorInvalidValue;
   // persistent grid when items are taken dynamically, else one CTA per item
   const int grid = a.work_ctr ? (a.grid < a.nitems ? a.grid : a.nitems) : a.nitems;

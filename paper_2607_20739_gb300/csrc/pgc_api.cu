@@ -40,6 +40,7 @@ struct Phase {
   std::vector<int64_t> e_row0, e_rows, e_zrow0;
   int64_t z_total = 0, max_rows = 0;
   int max_item_rows = 1;
+  int tail = 0;                         // fused tail of the gradient kernel
   // device copies
   WorkItem* d_items = nullptr;
   int32_t* d_e_item0 = nullptr;
@@ -342,6 +343,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   ctx->phases.resize(1 + ctx->c);
   build_phase(ctx, ctx->phases[0], -1);
   for (int o = 0; o < ctx->c; ++o) build_phase(ctx, ctx->phases[1 + o], o);
+  for (auto& ph : ctx->phases) ph.tail = ctx->loss == PGC_SOFTMAX ? 0 : ctx->tail_mode;
   size_t max_partials = 0;
   int64_t max_z = 0;
   for (auto& ph : ctx->phases) {
@@ -505,7 +507,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     g.X = ctx->X; g.y = static_cast<const float*>(ctx->y); g.w = ctx->w;
     g.items = ph.d_items; g.nitems = (int)ph.items.size(); g.max_item_rows = ph.max_item_rows;
     g.partials = ctx->partials; g.status = ctx->status;
-    g.tail = ctx->tail_mode; g.pdl = ctx->pdl;
+    g.tail = ph.tail; g.pdl = ctx->pdl;
     g.cnt_e = ctx->counters; g.cnt_all = ctx->counters + n;
     g.work_ctr = ctx->counters + n + 1; g.prod_done = ctx->counters + n + 2; g.grid = ctx->sm_count;
     g.e_item0 = ph.d_e_item0; g.e_scale = ph.d_e_scale; g.e_dest = ph.d_e_dest; g.ndest = ph.ndest;
@@ -513,7 +515,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     nl[PGC_KGRAD] = 1;
     PGC_CK(ctx, launch_grad_rows(g, ctx->variant, st));
     need_commit = false;
-    need_decode = ctx->tail_mode < 2;
+    need_decode = ph.tail < 2;
   } else {
     SoftmaxCCArgs a;
     a.dtype = ctx->dtype; a.ld = ctx->ld; a.K = ctx->K; a.X = ctx->X; a.y = static_cast<const int32_t*>(ctx->y);
