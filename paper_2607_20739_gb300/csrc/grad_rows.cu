@@ -93,6 +93,7 @@ struct Smem {
   uint64_t* sync;       // consumer barrier (count kNW)
   uint64_t* red_full;   // consumers -> tail warp (count kNW)
   uint64_t* red_free;   // tail warp -> consumers (count 1)
+  uint64_t* stage_sync; // CTA-per-row dot exchange (count kNW)
   Handoff* ho;
   DecodePlan* plan;     // decode coefficients (tail == 2), derived at kernel start
   StageHdr* hdr;
@@ -117,6 +118,7 @@ __device__ __forceinline__ Smem carve(uint8_t* base, const StageCfg& c, bool blo
   m.sync = m.empty + c.S;
   m.red_full = m.sync + 1;
   m.red_free = m.sync + 2;
+  m.stage_sync = m.sync + 3;
   off = a128(sizeof(uint64_t) * (2 * c.S + 4));
   m.ho = reinterpret_cast<Handoff*>(base + off);
   off = a128(off + sizeof(Handoff));
@@ -155,6 +157,22 @@ struct ConsumerSync {
     __syncwarp();                        // lane 0's acquire covers the whole warp
     bool ok = true;
     if (!last) ok = mbar_wait(bar, phase, status);
+    phase ^= 1u;
+    return __all_sync(0xffffffffu, ok);
+  }
+};
+
+// A plain barrier of the 8 consumer warps on its own mbarrier (count kNW),
+// bounded: used once per stage by the CTA-per-row consumers, where every
+// warp arrives at about the same time.
+struct StageSync {
+  uint64_t* bar;
+  uint32_t phase;
+  int* status;
+  __device__ __forceinline__ bool operator()() {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+    const bool ok = mbar_wait(bar, phase, status);
     phase ^= 1u;
     return __all_sync(0xffffffffu, ok);
   }
@@ -400,6 +418,7 @@ __device__ void consume_block_row(const GradRowsArgs& a, const Smem& sm, const S
   constexpr int E = NCH * VEC;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
   ConsumerSync bar{sm.sync, &sm.ho->sync_count, 0u, a.status};
+  StageSync xbar{sm.stage_sync, 0u, a.status};
   if (a.pdl) grid_dep_wait();
   float wr[E], acc[E];
 #pragma unroll
@@ -434,7 +453,7 @@ __device__ void consume_block_row(const GradRowsArgs& a, const Smem& sm, const S
     }
     // the exchange buffer alternates by stage parity; the barrier of stage
     // i + 1 separates this stage's reads from stage i + 2's writes
-    if (!bar()) { ok = false; break; }
+    if (!xbar()) { ok = false; break; }
     for (int rr = 0; rr < h.rows; ++rr) {
       float dot = 0.f;
 #pragma unroll
@@ -482,6 +501,7 @@ __global__ void __launch_bounds__(kThreads, 1) grad_rows_kernel(GradRowsArgs a, 
     mbar_init(sm.sync, kNW);
     mbar_init(sm.red_full, kNW);
     mbar_init(sm.red_free, 1);
+    mbar_init(sm.stage_sync, kNW);
     sm.ho->item = -1;
     sm.ho->e = -1;
     sm.ho->commit = -1;
