@@ -41,6 +41,15 @@ struct Phase {
   int64_t z_total = 0, max_rows = 0;
   int max_item_rows = 1;
   int tail = 0;                         // fused tail of the gradient kernel
+  // tensor-core softmax path: partitions' Z / R rows padded to 64
+  std::vector<int64_t> e_zrow0p;
+  std::vector<int32_t> f_prefix, f_nk, f_aoff, f_mvalid, b_prefix, b_nk, b_aoff, b_boff, b_mvalid;
+  std::vector<int64_t> f_outrow0;
+  int64_t zpad_total = 0;
+  int64_t* d_e_zrow0p = nullptr;
+  int32_t *d_f_prefix = nullptr, *d_f_nk = nullptr, *d_f_aoff = nullptr, *d_f_mvalid = nullptr;
+  int32_t *d_b_prefix = nullptr, *d_b_nk = nullptr, *d_b_aoff = nullptr, *d_b_boff = nullptr, *d_b_mvalid = nullptr;
+  int64_t* d_f_outrow0 = nullptr;
   // device copies
   WorkItem* d_items = nullptr;
   int32_t* d_e_item0 = nullptr;
@@ -102,6 +111,13 @@ struct pgc_ctx {
                              // work-item counter, finished producers (zero between steps)
   bool pdl = true;           // chain the step's kernels with programmatic dependent launch
   int tail_mode = 0;         // fused tail of the gradient kernel (see GradRowsArgs)
+  bool tc = false;           // softmax on the tensor cores (bf16 features)
+  int64_t Ktc = 0;           // classes padded to the forward N tile (256)
+  uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]
+  alignas(64) unsigned char tmXk[128];   // X as K-major A   (box 64 x 128)
+  alignas(64) unsigned char tmW[128];    // Wb as K-major B  (box 64 x 256)
+  alignas(64) unsigned char tmR[128];    // R as MN-major A  (box 64 x 64)
+  alignas(64) unsigned char tmXm[128];   // X as MN-major B  (box 64 x 64)
   int64_t loss_chunk = 0;
   int loss_nblocks = 256;
   void* tables = nullptr;
@@ -209,6 +225,28 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
     }
   } else {
     for (int e = 0; e <= nE; ++e) ph.e_item0.push_back(e);
+    if (ctx->tc) {
+      const int NTf = (int)(ctx->Ktc / 256), MTb = (int)(ctx->Ktc / 128), NTb = (int)(ctx->ld / 256);
+      int64_t zp = 0;
+      ph.f_prefix.push_back(0);
+      ph.b_prefix.push_back(0);
+      for (int e = 0; e < nE; ++e) {
+        const int64_t m = ph.e_rows[e];
+        ph.e_zrow0p.push_back(zp);
+        ph.f_nk.push_back((int32_t)(ctx->ld / 64));
+        ph.f_aoff.push_back((int32_t)ph.e_row0[e]);
+        ph.f_outrow0.push_back(zp);
+        ph.f_mvalid.push_back((int32_t)m);
+        ph.f_prefix.push_back(ph.f_prefix.back() + (int32_t)((m + 127) / 128) * NTf);
+        ph.b_nk.push_back((int32_t)((m + 63) / 64));
+        ph.b_aoff.push_back((int32_t)zp);
+        ph.b_boff.push_back((int32_t)ph.e_row0[e]);
+        ph.b_mvalid.push_back((int32_t)ctx->K);
+        ph.b_prefix.push_back(ph.b_prefix.back() + MTb * NTb);
+        zp += (m + 63) / 64 * 64;
+      }
+      ph.zpad_total = zp;
+    }
   }
 }
 
@@ -236,7 +274,7 @@ void free_all(pgc_ctx* ctx) {
   for (cudaEvent_t ev : ctx->ev_pool) cudaEventDestroy(ev);
   ctx->ev_pool.clear();
   void* ptrs[] = {ctx->X, ctx->y, ctx->w, ctx->wb, ctx->store, ctx->U, ctx->gout, ctx->partials, ctx->Z,
-                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->tables, ctx->counters};
+                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->tables, ctx->counters, ctx->Rb};
   for (void* p : ptrs)
     if (p) cudaFree(p);
 }
@@ -319,7 +357,11 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
     ctx->variant = grad_rows_variant(dtype, d, &ctx->ld);
     if (ctx->variant < 0) { delete ctx; return PGC_ENOTSUP; }
   } else {
-    ctx->ld = (int64_t)align_up((size_t)d, 64);
+    // bf16 softmax runs on the tensor cores (PGC_NO_TC=1 keeps the CUDA-core path)
+    const char* env = std::getenv("PGC_NO_TC");
+    ctx->tc = dtype == PGC_BF16 && K >= kTcMinClasses && !(env && env[0] == '1');
+    ctx->ld = (int64_t)align_up((size_t)d, ctx->tc ? 256 : 64);
+    ctx->Ktc = (int64_t)align_up((size_t)K, 256);
   }
   ctx->P = ctx->K * ctx->ld;
   ctx->Kpad = (int64_t)align_up((size_t)K, 4);
@@ -347,13 +389,17 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   size_t max_partials = 0;
   int64_t max_z = 0;
   for (auto& ph : ctx->phases) {
-    const size_t np = ctx->loss == PGC_SOFTMAX ? ph.parts.size() * (size_t)ctx->P : ph.items.size() * (size_t)ctx->ld;
+    // the tensor-core backward writes the stores directly: no partials
+    const size_t np = ctx->tc ? 0
+                      : ctx->loss == PGC_SOFTMAX ? ph.parts.size() * (size_t)ctx->P
+                                                 : ph.items.size() * (size_t)ctx->ld;
     max_partials = std::max(max_partials, np);
     max_z = std::max(max_z, ph.z_total);
   }
   std::vector<uint8_t> tab;
   size_t off = 0;
   std::vector<size_t> offs;
+  constexpr int kTabs = 18;
   for (auto& ph : ctx->phases) {
     offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
@@ -362,6 +408,17 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_row0);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_rows);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_zrow0);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.e_zrow0p);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.f_prefix);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.f_nk);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.f_aoff);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.f_mvalid);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.f_outrow0);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_prefix);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_nk);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_aoff);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_boff);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_mvalid);
   }
   // loss chunks (softmax): {row0, rows, 0} per chunk
   std::vector<int64_t> ldesc;
@@ -392,13 +449,20 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   PGC_ALLOC(ctx->X, (size_t)ctx->total_rows * ctx->ld * ctx->esize);
   PGC_ALLOC(ctx->y, (size_t)ctx->total_rows * 4 + 64);   // per-stage label copies overrun by <= 12 B
   PGC_ALLOC(ctx->w, Pb);
-  if (dtype == PGC_BF16) PGC_ALLOC(ctx->wb, (size_t)ctx->P * 2);
+  const size_t wb_elems = ctx->tc ? (size_t)ctx->Ktc * ctx->ld : (size_t)ctx->P;
+  if (dtype == PGC_BF16) PGC_ALLOC(ctx->wb, wb_elems * 2);
   PGC_ALLOC(ctx->store, (size_t)ctx->owners * ctx->c * Pb);
   PGC_ALLOC(ctx->U, (size_t)ctx->c * Pb);
   PGC_ALLOC(ctx->gout, Pb);
   PGC_ALLOC(ctx->partials, max_partials * sizeof(float));
-  if (loss == PGC_SOFTMAX)
-    PGC_ALLOC(ctx->Z, (size_t)std::max<int64_t>(max_z, ctx->loss_chunk) * ctx->Kpad * sizeof(float));
+  int64_t max_zpad = 0;
+  for (auto& ph : ctx->phases) max_zpad = std::max(max_zpad, ph.zpad_total);
+  if (loss == PGC_SOFTMAX) {
+    const size_t zcc = (size_t)std::max<int64_t>(max_z, ctx->loss_chunk) * ctx->Kpad;
+    const size_t ztc = ctx->tc ? (size_t)max_zpad * ctx->Ktc : 0;
+    PGC_ALLOC(ctx->Z, std::max(zcc, ztc) * sizeof(float));
+  }
+  if (ctx->tc) PGC_ALLOC(ctx->Rb, (size_t)max_zpad * ctx->Ktc * sizeof(uint16_t));
   PGC_ALLOC(ctx->coeff, (size_t)n * sizeof(float));
   PGC_ALLOC(ctx->status, sizeof(int));
   PGC_ALLOC(ctx->loss_blocks, (size_t)ctx->loss_nblocks * sizeof(double));
@@ -419,23 +483,45 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   if (e == cudaSuccess && w0)
     e = cudaMemcpy2DAsync(ctx->w, ctx->ld * sizeof(float), w0, d * sizeof(float), d * sizeof(float), K,
                           cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && ctx->wb) e = cudaMemsetAsync(ctx->wb, 0, wb_elems * 2, st);
   if (e == cudaSuccess && ctx->wb) e = launch_f32_to_bf16(ctx->w, ctx->wb, ctx->P, st);
+  if (e == cudaSuccess && ctx->Rb) e = cudaMemsetAsync(ctx->Rb, 0, (size_t)max_zpad * ctx->Ktc * 2, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return fail(e);
 
   uint8_t* base = static_cast<uint8_t*>(ctx->tables);
   for (size_t i = 0; i < ctx->phases.size(); ++i) {
     Phase& ph = ctx->phases[i];
-    ph.d_items = reinterpret_cast<WorkItem*>(base + offs[7 * i + 0]);
-    ph.d_e_item0 = reinterpret_cast<int32_t*>(base + offs[7 * i + 1]);
-    ph.d_e_scale = reinterpret_cast<float*>(base + offs[7 * i + 2]);
-    ph.d_e_dest = reinterpret_cast<int32_t*>(base + offs[7 * i + 3]);
-    ph.d_e_row0 = reinterpret_cast<int64_t*>(base + offs[7 * i + 4]);
-    ph.d_e_rows = reinterpret_cast<int64_t*>(base + offs[7 * i + 5]);
-    ph.d_e_zrow0 = reinterpret_cast<int64_t*>(base + offs[7 * i + 6]);
+    const size_t* o = &offs[kTabs * i];
+    ph.d_items = reinterpret_cast<WorkItem*>(base + o[0]);
+    ph.d_e_item0 = reinterpret_cast<int32_t*>(base + o[1]);
+    ph.d_e_scale = reinterpret_cast<float*>(base + o[2]);
+    ph.d_e_dest = reinterpret_cast<int32_t*>(base + o[3]);
+    ph.d_e_row0 = reinterpret_cast<int64_t*>(base + o[4]);
+    ph.d_e_rows = reinterpret_cast<int64_t*>(base + o[5]);
+    ph.d_e_zrow0 = reinterpret_cast<int64_t*>(base + o[6]);
+    ph.d_e_zrow0p = reinterpret_cast<int64_t*>(base + o[7]);
+    ph.d_f_prefix = reinterpret_cast<int32_t*>(base + o[8]);
+    ph.d_f_nk = reinterpret_cast<int32_t*>(base + o[9]);
+    ph.d_f_aoff = reinterpret_cast<int32_t*>(base + o[10]);
+    ph.d_f_mvalid = reinterpret_cast<int32_t*>(base + o[11]);
+    ph.d_f_outrow0 = reinterpret_cast<int64_t*>(base + o[12]);
+    ph.d_b_prefix = reinterpret_cast<int32_t*>(base + o[13]);
+    ph.d_b_nk = reinterpret_cast<int32_t*>(base + o[14]);
+    ph.d_b_aoff = reinterpret_cast<int32_t*>(base + o[15]);
+    ph.d_b_boff = reinterpret_cast<int32_t*>(base + o[16]);
+    ph.d_b_mvalid = reinterpret_cast<int32_t*>(base + o[17]);
   }
   ctx->loss_desc = nullptr;
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
+  if (ctx->tc) {
+    const uint64_t pitch = (uint64_t)ctx->ld * 2;
+    bool ok = make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, 128) &&
+              make_tmap_bf16(ctx->tmW, ctx->wb, ctx->ld, ctx->Ktc, pitch, 256) &&
+              make_tmap_bf16(ctx->tmR, ctx->Rb, ctx->Ktc, max_zpad, (uint64_t)ctx->Ktc * 2, 64) &&
+              make_tmap_bf16(ctx->tmXm, ctx->X, ctx->ld, ctx->total_rows, pitch, 64);
+    if (!ok) return fail(cudaErrorInvalidValue);
+  }
 #undef PGC_ALLOC
   *out = ctx;
   return PGC_OK;
@@ -516,6 +602,27 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     PGC_CK(ctx, launch_grad_rows(g, ctx->variant, st));
     need_commit = false;
     need_decode = ph.tail < 2;
+  } else if (ctx->tc) {
+    // tensor cores: Z = X Wb^T, R = softmax(Z) - onehot(y) in bf16, then
+    // G_e = (1/m_e) R_e^T X_e written straight into the stores
+    const int nE = (int)ph.parts.size();
+    TcGemmParams f = {};
+    f.nbatch = nE; f.tile_prefix = ph.d_f_prefix; f.NT = (int)(ctx->Ktc / 256); f.nk = ph.d_f_nk;
+    f.a_off = ph.d_f_aoff; f.b_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back(); f.backward = 0;
+    f.out = ctx->Z; f.out_ld = ctx->Ktc; f.out_row0 = ph.d_f_outrow0; f.m_valid = ph.d_f_mvalid;
+    f.n_valid = (int)ctx->Ktc; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
+    PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, f, false, false, ctx->sm_count, st));
+    PGC_CK(ctx, launch_softmax_bf16(ctx->Z, ctx->Rb, ctx->Ktc, ctx->K, static_cast<const int32_t*>(ctx->y),
+                                    ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows, false, st));
+    TcGemmParams b = {};
+    b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
+    b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff; b.total_tiles = ph.b_prefix.back(); b.backward = 1;
+    b.out = ctx->store; b.out_ld = ctx->ld; b.m_valid = ph.d_b_mvalid; b.n_valid = (int)ctx->ld;
+    b.scale = ph.d_e_scale; b.dest = ph.d_e_dest; b.ndest = ph.ndest; b.dest_stride = ctx->P;
+    b.status = ctx->status; b.pdl = ctx->pdl ? 1 : 0;
+    PGC_CK(ctx, launch_tc_gemm(ctx->tmR, ctx->tmXm, b, true, true, ctx->sm_count, st));
+    nl[PGC_KGRAD] = 3;
+    need_commit = false;
   } else {
     SoftmaxCCArgs a;
     a.dtype = ctx->dtype; a.ld = ctx->ld; a.K = ctx->K; a.X = ctx->X; a.y = static_cast<const int32_t*>(ctx->y);

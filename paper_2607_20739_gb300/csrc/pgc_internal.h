@@ -26,6 +26,9 @@ struct WorkItem {
 
 // ---- K5 + K6: decode coefficients from the mask, decode, SGD --------------
 constexpr int kMaxWorkers = 1024;
+// softmax on the tensor cores from this many classes on (the forward N tile is
+// 256 classes; below half a tile the padding outweighs the tensor-core gain)
+constexpr int64_t kTcMinClasses = 128;
 struct MaskBits {
   uint32_t w[kMaxWorkers / 32];
 };
@@ -148,6 +151,40 @@ struct LossArgs {
   const int64_t* chunk_desc; // device [3 * nchunks]: {row0, rows, 0} per chunk
 };
 cudaError_t launch_loss(const LossArgs& a, cudaStream_t st);
+
+// ---- tensor-core softmax gradient (tc_gemm.cu) ---------------------------
+// forward  Z[r][k] = sum_j X[r][j] Wb[k][j]   (A = X K-major, B = Wb K-major)
+// backward G_e[k][j] = scale_e sum_r R[r][k] X[r][j]  (A = R MN-major, B = X MN-major)
+struct TcGemmParams {
+  int nbatch;
+  const int* tile_prefix;   // [nbatch + 1] tiles before batch b (MT_b * NT each)
+  int NT;                   // N tiles (of 256) per batch
+  const int* nk;            // [nbatch] K blocks (of 64)
+  const int* a_off;         // [nbatch] A row offset (K-major: M rows; MN-major: K rows)
+  const int* b_off;         // [nbatch] B row offset (MN-major: K rows)
+  int total_tiles;
+  int backward;             // 0: forward -> Z rows, 1: backward -> stores
+  float* out;
+  int64_t out_ld;           // floats between output rows
+  const int64_t* out_row0;  // forward: first Z row of batch b
+  const int* m_valid;       // [nbatch] output rows that exist
+  int n_valid;              // output columns that exist
+  const float* scale;       // backward: 1/m_e
+  const int32_t* dest;      // backward: [nbatch * ndest] store index or -1
+  int ndest;
+  int64_t dest_stride;      // floats per store
+  int* status;
+  int pdl;
+};
+// tm_out: 128 bytes, 64-byte aligned (a CUtensorMap)
+bool make_tmap_bf16(void* tm_out, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+                    uint32_t box_outer);
+cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const TcGemmParams& p, bool a_mn, bool b_mn, int grid,
+                           cudaStream_t st);
+// R = softmax(Z) - onehot(y) as bf16, zero for classes K..Kpad-1
+cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int64_t K, const int32_t* y,
+                                const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
+                                int64_t max_rows, bool pdl, cudaStream_t st);
 
 // ---- misc -------------------------------------------------------------------
 cudaError_t launch_f32_to_bf16(const float* src, uint16_t* dst, int64_t count, cudaStream_t st);

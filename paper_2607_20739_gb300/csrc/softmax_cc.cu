@@ -145,6 +145,54 @@ __global__ void __launch_bounds__(256) backward_tiled(const T* __restrict__ X, i
   }
 }
 
+// R = softmax(Z) - onehot(y) written as bf16 for the tensor-core backward;
+// one warp per row of an evaluated partition, zero for the padded classes.
+__global__ void softmax_residual_bf16(const float* __restrict__ Z, uint16_t* __restrict__ Rb, int64_t Kpad, int64_t K,
+                                      const int32_t* __restrict__ y, const int64_t* e_row0, const int64_t* e_rows,
+                                      const int64_t* e_zrow0) {
+  const int e = blockIdx.y;
+  const int lane = threadIdx.x & 31;
+  const int64_t rows = e_rows[e];
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  // rows up to the next multiple of 64 are the backward GEMM's K padding: they
+  // are written as zeros, since another phase may have left values there
+  const int64_t rows_pad = (rows + 63) / 64 * 64;
+  for (int64_t r = warp; r < rows_pad; r += nwarps) {
+    const int64_t zr = e_zrow0[e] + r;
+    uint16_t* out = Rb + zr * Kpad;
+    if (r >= rows) {
+      for (int64_t k = lane; k < Kpad; k += 32) out[k] = 0;
+      continue;
+    }
+    const float* z = Z + zr * Kpad;
+    float m = -INFINITY;
+    for (int64_t k = lane; k < K; k += 32) m = fmaxf(m, z[k]);
+    m = warp_max(m);
+    float sum = 0.f;
+    for (int64_t k = lane; k < K; k += 32) sum += expf(z[k] - m);
+    sum = warp_sum(sum);
+    const float inv = 1.0f / sum;
+    const int lab = y[e_row0[e] + r];
+    for (int64_t k = lane; k < Kpad; k += 32) {
+      const float v = k < K ? expf(z[k] - m) * inv - (k == lab ? 1.0f : 0.0f) : 0.0f;
+      __nv_bfloat16 bv = __float2bfloat16_rn(v);
+      out[k] = *reinterpret_cast<uint16_t*>(&bv);
+    }
+  }
+}
+
+cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int64_t K, const int32_t* y,
+                                const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
+                                int64_t max_rows, bool pdl, cudaStream_t st) {
+  (void)pdl;
+  if (nE <= 0) return cudaSuccess;
+  int64_t bx = ((max_rows + 63) / 64 * 64 * 32 + 255) / 256;
+  if (bx > 512) bx = 512;
+  softmax_residual_bf16<<<dim3((unsigned)bx, (unsigned)nE), 256, 0, st>>>(Z, Rb, Kpad, K, y, e_row0, e_rows, e_zrow0);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_softmax_cc(const SoftmaxCCArgs& a, cudaStream_t st) {
   if (a.nE <= 0) return cudaSuccess;
   const dim3 g1((unsigned)((a.K + TB - 1) / TB), (unsigned)((a.max_rows + TB - 1) / TB), (unsigned)a.nE);

@@ -1,0 +1,354 @@
+// Tensor-core GEMMs of the softmax gradient (§III with f = log sum_k exp(w_k.x)
+// - w_y.x), on the sm_103a tcgen05 path:
+//
+//   forward   Z[r][k]   = sum_j X[r][j] W[k][j]                 A = X (K-major),  B = W (K-major)
+//   backward  G_e[k][j] = (1/m_e) sum_{r in D_e} R[r][k] X[r][j]  A = R (MN-major), B = X (MN-major)
+//
+// with R = softmax(Z) - onehot(y) in bf16 between them.  Both are one
+// persistent, warp-specialised kernel: warp 0 streams 128x64 A tiles and
+// 256x64 B tiles into a 4-stage shared-memory ring with 2-D TMA
+// (cp.async.bulk.tensor, 128-byte swizzle), warp 1 issues
+// tcgen05.mma.cta_group::1.kind::f16 (bf16 in, fp32 accumulate) into one of
+// two 128x256 TMEM accumulators, and warps 2-5 drain the other accumulator
+// with tcgen05.ld and write fp32 results (forward: logits; backward: the new
+// gradient straight into every store that keeps it, scaled by 1/m_e).
+// Every wait is bounded; the TMEM allocation is released on every path.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+
+#include "tail.cuh"
+
+namespace pgc {
+
+constexpr int kTM = 128, kTN = 256, kTK = 64;
+constexpr int kGStages = 4;
+constexpr uint32_t kABytes = kTM * kTK * 2;    // 16 KB
+constexpr uint32_t kBBytes = kTN * kTK * 2;    // 32 KB
+constexpr int kGemmThreads = 192;              // producer, MMA, 4 epilogue warps
+constexpr uint32_t kTmemCols = 2 * kTN;        // two fp32 accumulators
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"(tm), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Shared-memory matrix descriptor of a tcgen05 operand in the canonical
+// 128-byte-swizzled layout: start address, leading and stride byte offsets
+// (16-byte units), descriptor version 1, swizzle mode 2 (128 B).
+__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+
+// Instruction descriptor of kind::f16: fp32 accumulator (bits 4-5 = 1),
+// bf16 A and B (bits 7-9, 10-12 = 1), operand majorness (bits 15, 16),
+// N >> 3 (bits 17-22), M >> 4 (bits 24-28).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool a_mn, bool b_mn) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) | ((b_mn ? 1u : 0u) << 16) |
+         ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_bf16(uint32_t tmem_d, uint64_t da, uint64_t db, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(da), "l"(db), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
+// the kernel
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void decode_tile(const TcGemmParams& p, int t, int& b, int& mt, int& nt) {
+  int lo = 0, hi = p.nbatch - 1;
+  while (lo < hi) {                      // last b with tile_prefix[b] <= t
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.tile_prefix[mid] <= t) lo = mid; else hi = mid - 1;
+  }
+  b = lo;
+  const int rem = t - p.tile_prefix[b];
+  mt = rem / p.NT;
+  nt = rem % p.NT;
+}
+
+template <bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcGemmParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kGStages * kABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kGStages * kBBytes);
+  uint64_t* empty = full + kGStages;
+  uint64_t* acc_full = empty + kGStages;
+  uint64_t* acc_empty = acc_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  __shared__ int cta_err;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    cta_err = 0;
+    for (int s = 0; s < kGStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 4);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  if (threadIdx.x == 0) grid_dep_launch();
+  if (p.pdl) grid_dep_wait();           // inputs are the previous kernels' outputs
+
+  // tiles of this CTA: blockIdx.x, blockIdx.x + gridDim.x, ...
+  const int my_tiles = p.total_tiles > (int)blockIdx.x
+                           ? (p.total_tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x
+                           : 0;
+
+  if (warp == 0 && lane == 0) {
+    // ---- producer ----------------------------------------------------------
+    int it = 0;
+    bool ok = true;
+    for (int i = 0; i < my_tiles && ok; ++i) {
+      int b, mt, nt;
+      decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
+      const int nkb = p.nk[b];
+      for (int kb = 0; kb < nkb; ++kb, ++it) {
+        const int s = it % kGStages;
+        if (it >= kGStages && !mbar_wait(&empty[s], ((it / kGStages) - 1) & 1, p.status)) { ok = false; break; }
+        mbar_arrive_expect_tx(&full[s], kABytes + kBBytes);
+        uint8_t* a_dst = sA + (size_t)s * kABytes;
+        uint8_t* b_dst = sB + (size_t)s * kBBytes;
+        if (!A_MN) {
+          tma_load_2d(a_dst, &tmA, kb * kTK, p.a_off[b] + mt * kTM, &full[s]);
+        } else {
+          for (int j = 0; j < kTM / 64; ++j)
+            tma_load_2d(a_dst + j * 8192, &tmA, mt * kTM + j * 64, p.a_off[b] + kb * kTK, &full[s]);
+        }
+        if (!B_MN) {
+          tma_load_2d(b_dst, &tmB, kb * kTK, nt * kTN, &full[s]);
+        } else {
+          for (int j = 0; j < kTN / 64; ++j)
+            tma_load_2d(b_dst + j * 8192, &tmB, nt * kTN + j * 64, p.b_off[b] + kb * kTK, &full[s]);
+        }
+      }
+    }
+    if (!ok) atomicExch(&cta_err, 1);
+    // no copy may outlive the CTA: wait for the last fill of every stage
+    for (int s = 0; s < kGStages && s < it; ++s) {
+      const int last = ((it - 1 - s) / kGStages) * kGStages + s;
+      mbar_wait(&full[s], (last / kGStages) & 1, p.status);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer --------------------------------------------------------
+    constexpr uint32_t idesc = idesc_bf16_f32(kTM, kTN, A_MN, B_MN);
+    int it = 0;
+    bool ok = true;
+    for (int i = 0; i < my_tiles && ok; ++i) {
+      int b, mt, nt;
+      decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
+      const int acc = i & 1;
+      if (i >= 2 && !mbar_wait(&acc_empty[acc], ((i / 2) - 1) & 1, p.status)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem + (uint32_t)(acc * kTN);
+      const int nkb = p.nk[b];
+      for (int kb = 0; kb < nkb; ++kb, ++it) {
+        const int s = it % kGStages;
+        if (!mbar_wait(&full[s], (it / kGStages) & 1, p.status)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t a_base = smem_u32(sA + (size_t)s * kABytes);
+        const uint32_t b_base = smem_u32(sB + (size_t)s * kBBytes);
+#pragma unroll
+        for (int kk = 0; kk < kTK / 16; ++kk) {
+          // K-major: the next 16 K elements are 32 bytes further along each
+          // 128-byte row; MN-major: 16 K rows further, 2 groups of 8 rows.
+          const uint64_t da = A_MN ? smem_desc_sw128(a_base + kk * 2048, 8192, 1024)
+                                   : smem_desc_sw128(a_base + kk * 32, 16, 1024);
+          const uint64_t db = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
+                                   : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+          umma_bf16(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
+        }
+        umma_commit(&empty[s]);          // the stage is free once these MMAs finish
+      }
+      if (!ok) break;
+      umma_commit(&acc_full[acc]);       // the accumulator is complete
+    }
+    if (!ok) atomicExch(&cta_err, 1);
+  } else if (warp >= 2) {
+    // ---- epilogue ----------------------------------------------------------
+    const int q = warp & 3;              // TMEM lane quarter this warp may read
+    const int row_in_tile = q * 32 + lane;
+    for (int i = 0; i < my_tiles; ++i) {
+      int b, mt, nt;
+      decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
+      const int acc = i & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[acc], (i / 2) & 1, p.status))) {
+        atomicExch(&cta_err, 1);
+        break;
+      }
+      tc_fence_after();
+      const int m = mt * kTM + row_in_tile;
+      const bool mvalid = m < p.m_valid[b];
+      const uint32_t t_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTN);
+      for (int ch = 0; ch < kTN / 32; ++ch) {
+        uint32_t r[32];
+        tmem_ld32(t_base + ch * 32, r);
+        tmem_ld_wait();
+        const int n0 = nt * kTN + ch * 32;
+        if (!mvalid || n0 >= p.n_valid) continue;
+        if (!p.backward) {
+          float4* dst = reinterpret_cast<float4*>(p.out + (p.out_row0[b] + m) * p.out_ld + n0);
+#pragma unroll
+          for (int v = 0; v < 8; ++v)
+            dst[v] = make_float4(__uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1]),
+                                 __uint_as_float(r[4 * v + 2]), __uint_as_float(r[4 * v + 3]));
+        } else {
+          const float sc = p.scale[b];
+          for (int k = 0; k < p.ndest; ++k) {
+            const int dd = p.dest[(int64_t)b * p.ndest + k];
+            if (dd < 0) continue;
+            float4* dst = reinterpret_cast<float4*>(p.out + (int64_t)dd * p.dest_stride + (int64_t)m * p.out_ld + n0);
+#pragma unroll
+            for (int v = 0; v < 8; ++v)
+              dst[v] = make_float4(sc * __uint_as_float(r[4 * v]), sc * __uint_as_float(r[4 * v + 1]),
+                                   sc * __uint_as_float(r[4 * v + 2]), sc * __uint_as_float(r[4 * v + 3]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[acc]);
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    // every MMA of this CTA has completed before its accumulator was drained;
+    // after a failure, wait (bounded) for the last commits before releasing
+    if (cta_err && lane == 0) {
+      for (int a = 0; a < 2 && a < my_tiles; ++a) {
+        const int last = ((my_tiles - 1 - a) / 2) * 2 + a;
+        mbar_wait(&acc_full[a], (last / 2) & 1, p.status);
+      }
+    }
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return nullptr;
+    fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor map: [outer][inner] row-major, row pitch in bytes,
+// box {64, box_outer}, 128-byte swizzle; out-of-range elements read as zero.
+bool make_tmap_bf16(void* tm_out, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+                    uint32_t box_outer) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch_bytes};
+  cuuint32_t box[2] = {64, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(reinterpret_cast<CUtensorMap*>(tm_out), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+static size_t gemm_smem_bytes() {
+  return 1024 + kGStages * (size_t)(kABytes + kBBytes) + sizeof(uint64_t) * (2 * kGStages + 4) + 16;
+}
+
+template <bool A_MN, bool B_MN>
+static cudaError_t launch_tc(const void* tmA, const void* tmB, const TcGemmParams& p, int grid, cudaStream_t st) {
+  auto kern = tc_gemm_kernel<A_MN, B_MN>;
+  const size_t smem = gemm_smem_bytes();
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = p.pdl ? 1 : 0;
+  CUtensorMap a, b;
+  std::memcpy(&a, tmA, sizeof(CUtensorMap));
+  std::memcpy(&b, tmB, sizeof(CUtensorMap));
+  return cudaLaunchKernelEx(&cfg, kern, a, b, p);
+}
+
+cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const TcGemmParams& p, bool a_mn, bool b_mn, int grid,
+                           cudaStream_t st) {
+  if (p.total_tiles <= 0) return cudaSuccess;
+  if (grid > p.total_tiles) grid = p.total_tiles;
+  if (!a_mn && !b_mn) return launch_tc<false, false>(tmA, tmB, p, grid, st);
+  if (a_mn && b_mn) return launch_tc<true, true>(tmA, tmB, p, grid, st);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace pgc

@@ -35,6 +35,11 @@ CASES = {
     "cr_bf16_lsq_long_rows": (WL["cr_n64_lsq_d16384"].replace(n=4, s=1, dtype="bf16", d=9000, m=20), 5),
     "cr_f32_softmax_k3": (WL["cr_n128_softmax_k1000"].replace(n=4, s=1, dtype="f32", K=3, d=50, m=30), 6),
     "fr_bf16_softmax_k2": (WL["fr_n32_softmax_k10"].replace(n=4, s=1, K=2, d=70, m=65), 6),
+    # tensor-core softmax: ragged class, feature and row tiles
+    "cr_tc_k300_d320_m200": (WL["cr_n128_softmax_k1000"].replace(n=4, s=1, K=300, d=320, m=200), 5),
+    "fr_tc_k256_unequal_rows": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=256, d=600,
+                                                                     m=(130, 1, 64, 257)), 5),
+    "cr_tc_k128_c_equals_n": (WL["cr_n128_softmax_k1000"].replace(n=3, s=2, K=128, d=256, m=300), 5),
 }
 
 
