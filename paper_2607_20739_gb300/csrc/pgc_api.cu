@@ -118,6 +118,9 @@ struct pgc_ctx {
   alignas(64) unsigned char tmW[128];    // Wb as K-major B  (box 64 x 256)
   alignas(64) unsigned char tmR[128];    // R as MN-major A  (box 64 x 64)
   alignas(64) unsigned char tmXm[128];   // X as MN-major B  (box 64 x 64)
+  alignas(64) unsigned char tmZo[128];   // Z fp32 output     (box 32 x 32)
+  alignas(64) unsigned char tmSo[128];   // stores [slot][K][ld] fp32 output (box 32 x 32 x 1)
+  alignas(64) unsigned char tmUo[128];   // U [c][K][ld] fp32, reduce-add target
   int64_t loss_chunk = 0;
   int loss_nblocks = 256;
   void* tables = nullptr;
@@ -243,7 +246,7 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
         ph.b_boff.push_back((int32_t)ph.e_row0[e]);
         ph.b_mvalid.push_back((int32_t)ctx->K);
         ph.b_prefix.push_back(ph.b_prefix.back() + MTb * NTb);
-        zp += (m + 63) / 64 * 64;
+        zp += (m + 127) / 128 * 128;   // whole forward tiles: their TMA stores stay inside the partition
       }
       ph.zpad_total = zp;
     }
@@ -520,6 +523,12 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
               make_tmap_bf16(ctx->tmW, ctx->wb, ctx->ld, ctx->Ktc, pitch, 256) &&
               make_tmap_bf16(ctx->tmR, ctx->Rb, ctx->Ktc, max_zpad, (uint64_t)ctx->Ktc * 2, 64) &&
               make_tmap_bf16(ctx->tmXm, ctx->X, ctx->ld, ctx->total_rows, pitch, 64);
+    const uint64_t zd[2] = {(uint64_t)ctx->Ktc, (uint64_t)max_zpad}, zs[1] = {(uint64_t)ctx->Ktc * 4};
+    const uint64_t sd[3] = {(uint64_t)ctx->ld, (uint64_t)ctx->K, (uint64_t)ctx->owners * ctx->c};
+    const uint64_t ud[3] = {(uint64_t)ctx->ld, (uint64_t)ctx->K, (uint64_t)ctx->c};
+    const uint64_t ss[2] = {(uint64_t)ctx->ld * 4, (uint64_t)ctx->P * 4};
+    ok = ok && make_tmap_f32_box32(ctx->tmZo, ctx->Z, 2, zd, zs) && make_tmap_f32_box32(ctx->tmSo, ctx->store, 3, sd, ss) &&
+         make_tmap_f32_box32(ctx->tmUo, ctx->U, 3, ud, ss);
     if (!ok) return fail(cudaErrorInvalidValue);
   }
 #undef PGC_ALLOC
@@ -608,19 +617,24 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     const int nE = (int)ph.parts.size();
     TcGemmParams f = {};
     f.nbatch = nE; f.tile_prefix = ph.d_f_prefix; f.NT = (int)(ctx->Ktc / 256); f.nk = ph.d_f_nk;
+    // in steady phases every evaluated partition has one store at slot o_t,
+    // so the backward also forms U[o_t] = sum_e g_e (TMA reduce-add) and the
+    // decode reads it instead of re-summing the stores
+    const bool u_red = ph.slot >= 0 && ph.ndest == 1;
     f.a_off = ph.d_f_aoff; f.b_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back(); f.backward = 0;
-    f.out = ctx->Z; f.out_ld = ctx->Ktc; f.out_row0 = ph.d_f_outrow0; f.m_valid = ph.d_f_mvalid;
-    f.n_valid = (int)ctx->Ktc; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
-    PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, f, false, false, ctx->sm_count, st));
+    f.out_row0 = ph.d_f_outrow0; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
+    PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, ctx->tmZo, nullptr, f, false, false, ctx->sm_count, st));
     PGC_CK(ctx, launch_softmax_bf16(ctx->Z, ctx->Rb, ctx->Ktc, ctx->K, static_cast<const int32_t*>(ctx->y),
-                                    ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows, false, st));
+                                    ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows,
+                                    u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr, ctx->P, st));
     TcGemmParams b = {};
     b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
     b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff; b.total_tiles = ph.b_prefix.back(); b.backward = 1;
-    b.out = ctx->store; b.out_ld = ctx->ld; b.m_valid = ph.d_b_mvalid; b.n_valid = (int)ctx->ld;
-    b.scale = ph.d_e_scale; b.dest = ph.d_e_dest; b.ndest = ph.ndest; b.dest_stride = ctx->P;
+    b.scale = ph.d_e_scale; b.dest = ph.d_e_dest; b.ndest = ph.ndest; b.m_limit = (int)ctx->K;
+    b.u_reduce = u_red ? 1 : 0; b.u_slot = ph.slot;
     b.status = ctx->status; b.pdl = ctx->pdl ? 1 : 0;
-    PGC_CK(ctx, launch_tc_gemm(ctx->tmR, ctx->tmXm, b, true, true, ctx->sm_count, st));
+    PGC_CK(ctx, launch_tc_gemm(ctx->tmR, ctx->tmXm, ctx->tmSo, ctx->tmUo, b, true, true, ctx->sm_count, st));
+    dc.u_ready = u_red ? 1 : 0;
     nl[PGC_KGRAD] = 3;
     need_commit = false;
   } else {

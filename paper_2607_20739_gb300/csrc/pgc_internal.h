@@ -48,6 +48,7 @@ struct DecodeArgs {
   int* status;
   float* g_user = nullptr;  // optional extra destinations of ghat and beta, same
   float* w_user = nullptr;  // unpadded layout (used when ld == d)
+  int u_ready = 0;          // U[slot] already holds this step's slot total
 };
 // ---- K1: streaming gradient of logistic / least-squares partitions -------
 // For every work item: partial[item][0:ld] = sum over its rows x of
@@ -164,27 +165,36 @@ struct TcGemmParams {
   const int* b_off;         // [nbatch] B row offset (MN-major: K rows)
   int total_tiles;
   int backward;             // 0: forward -> Z rows, 1: backward -> stores
-  float* out;
-  int64_t out_ld;           // floats between output rows
-  const int64_t* out_row0;  // forward: first Z row of batch b
-  const int* m_valid;       // [nbatch] output rows that exist
-  int n_valid;              // output columns that exist
+  // Results leave through TMA stores of 32 x 32 fp32 boxes.  Forward: the
+  // output map is Z [rows][Kpad] (2-D), box at (n, out_row0[b] + m).
+  // Backward: the output map is the stores [slot][K][ld] (3-D), box at
+  // (n, m, dest) for every dest >= 0, scaled by scale[b]; with u_reduce the
+  // same box is also added (TMA reduce-add) into U [c][K][ld] at u_slot.
+  const int64_t* out_row0;  // forward: first Z row of batch b (a multiple of 128)
   const float* scale;       // backward: 1/m_e
   const int32_t* dest;      // backward: [nbatch * ndest] store index or -1
   int ndest;
-  int64_t dest_stride;      // floats per store
+  int u_reduce;
+  int u_slot;
+  int m_limit;              // backward: output rows that exist (K); boxes past it are skipped
   int* status;
   int pdl;
 };
-// tm_out: 128 bytes, 64-byte aligned (a CUtensorMap)
+// Tensor maps (tm_out: 128 bytes, 64-byte aligned, a CUtensorMap), 128-byte
+// swizzle, out-of-range elements read as zero and are not written.
+// bf16 2-D [outer][inner], box {64, box_outer}
 bool make_tmap_bf16(void* tm_out, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
                     uint32_t box_outer);
-cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const TcGemmParams& p, bool a_mn, bool b_mn, int grid,
-                           cudaStream_t st);
-// R = softmax(Z) - onehot(y) as bf16, zero for classes K..Kpad-1
+// fp32 rank-2 or rank-3 (dims innermost first, byte strides of dims 1..), box {32, 32, 1}
+bool make_tmap_f32_box32(void* tm_out, const void* base, int rank, const uint64_t* dims, const uint64_t* strides);
+cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, const void* tmU, const TcGemmParams& p,
+                           bool a_mn, bool b_mn, int grid, cudaStream_t st);
+// R = softmax(Z) - onehot(y) as bf16, zero for classes K..Kpad-1 and for the
+// rows up to the next multiple of 64; also zeroes zero_buf[0:zero_n] (floats,
+// a multiple of 4) when given.
 cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int64_t K, const int32_t* y,
                                 const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
-                                int64_t max_rows, bool pdl, cudaStream_t st);
+                                int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st);
 
 // ---- misc -------------------------------------------------------------------
 cudaError_t launch_f32_to_bf16(const float* src, uint16_t* dst, int64_t count, cudaStream_t st);

@@ -149,8 +149,13 @@ __global__ void __launch_bounds__(256) backward_tiled(const T* __restrict__ X, i
 // one warp per row of an evaluated partition, zero for the padded classes.
 __global__ void softmax_residual_bf16(const float* __restrict__ Z, uint16_t* __restrict__ Rb, int64_t Kpad, int64_t K,
                                       const int32_t* __restrict__ y, const int64_t* e_row0, const int64_t* e_rows,
-                                      const int64_t* e_zrow0) {
+                                      const int64_t* e_zrow0, float* zero_buf, int64_t zero_n4) {
   const int e = blockIdx.y;
+  if (zero_buf) {
+    const int64_t nthr = (int64_t)gridDim.x * gridDim.y * blockDim.x;
+    const int64_t tid = ((int64_t)blockIdx.y * gridDim.x + blockIdx.x) * blockDim.x + threadIdx.x;
+    for (int64_t i = tid; i < zero_n4; i += nthr) reinterpret_cast<float4*>(zero_buf)[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   const int lane = threadIdx.x & 31;
   const int64_t rows = e_rows[e];
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -184,12 +189,12 @@ __global__ void softmax_residual_bf16(const float* __restrict__ Z, uint16_t* __r
 
 cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int64_t K, const int32_t* y,
                                 const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
-                                int64_t max_rows, bool pdl, cudaStream_t st) {
-  (void)pdl;
+                                int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st) {
   if (nE <= 0) return cudaSuccess;
   int64_t bx = ((max_rows + 63) / 64 * 64 * 32 + 255) / 256;
   if (bx > 512) bx = 512;
-  softmax_residual_bf16<<<dim3((unsigned)bx, (unsigned)nE), 256, 0, st>>>(Z, Rb, Kpad, K, y, e_row0, e_rows, e_zrow0);
+  softmax_residual_bf16<<<dim3((unsigned)bx, (unsigned)nE), 256, 0, st>>>(Z, Rb, Kpad, K, y, e_row0, e_rows, e_zrow0,
+                                                                          zero_buf, zero_n / 4);
   return cudaGetLastError();
 }
 

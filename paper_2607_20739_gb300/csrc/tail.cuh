@@ -160,7 +160,7 @@ __device__ __forceinline__ void decode_columns(const DecodeArgs& a, const Decode
   const int ndev = pl.ndev;
   const float4* store = reinterpret_cast<const float4*>(a.store);
   float4* U = reinterpret_cast<float4*>(a.U);
-  const bool small = a.owners <= kMaxO && c <= kMaxC && ndev <= kMaxD && a.slot >= 0;
+  const bool small = a.owners <= kMaxO && c <= kMaxC && ndev <= kMaxD && a.slot >= 0 && !a.u_ready;
   for (int64_t p = tid; p < P4; p += nthr) {
     float4 V = f4zero(), D = f4zero();
     if (small) {
@@ -191,7 +191,7 @@ __device__ __forceinline__ void decode_columns(const DecodeArgs& a, const Decode
       }
     } else {
       for (int o = 0; o < c; ++o) {
-        if (a.slot < 0 || o == a.slot) {
+        if (a.slot < 0 || (o == a.slot && !a.u_ready)) {
           float4 u = f4zero();
           for (int r = 0; r < a.owners; ++r) u = f4add(u, __ldcg(store + ((int64_t)r * c + o) * P4 + p));
           U[(int64_t)o * P4 + p] = u;
@@ -235,7 +235,7 @@ __device__ void decode_chunks(const DecodeArgs& a, const DecodePlan& pl, float4 
     const bool inb = p < P4;
     float4 V = f4zero();
     for (int o = 0; o < c; ++o) {
-      if (a.slot < 0 || o == a.slot) {
+      if (a.slot < 0 || (o == a.slot && !a.u_ready)) {
         float4 part = f4zero();
         if (inb)
           for (int r = y; r < a.owners; r += kDecY) part = f4add(part, __ldcg(store + ((int64_t)r * c + o) * P4 + p));

@@ -10,8 +10,10 @@
 // (cp.async.bulk.tensor, 128-byte swizzle), warp 1 issues
 // tcgen05.mma.cta_group::1.kind::f16 (bf16 in, fp32 accumulate) into one of
 // two 128x256 TMEM accumulators, and warps 2-5 drain the other accumulator
-// with tcgen05.ld and write fp32 results (forward: logits; backward: the new
-// gradient straight into every store that keeps it, scaled by 1/m_e).
+// with tcgen05.ld, stage 32 x 32 fp32 boxes in (swizzled) shared memory and
+// write them with TMA stores (forward: logits; backward: the new gradient
+// straight into every store that keeps it, scaled by 1/m_e, and optionally
+// added into the slot total U[o_t] with a TMA reduce-add).
 // Every wait is bounded; the TMEM allocation is released on every path.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -28,6 +30,8 @@ constexpr uint32_t kABytes = kTM * kTK * 2;    // 16 KB
 constexpr uint32_t kBBytes = kTN * kTK * 2;    // 32 KB
 constexpr int kGemmThreads = 192;              // producer, MMA, 4 epilogue warps
 constexpr uint32_t kTmemCols = 2 * kTN;        // two fp32 accumulators
+constexpr uint32_t kStageBox = 32 * 32 * 4;    // one 32 x 32 fp32 output box
+constexpr uint32_t kEpiBytes = 4 * 2 * kStageBox;  // two boxes per epilogue warp
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
@@ -38,6 +42,29 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, in
           smem_u32(dst)),
       "l"(tm), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(tm), "r"(x),
+               "r"(y), "r"(smem_u32(src))
+               : "memory");
+}
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, const void* src, int x, int y, int z) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(tm), "r"(x),
+               "r"(y), "r"(z), "r"(smem_u32(src))
+               : "memory");
+}
+__device__ __forceinline__ void tma_reduce_add_3d(const CUtensorMap* tm, const void* src, int x, int y, int z) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.3d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(tm),
+      "r"(x), "r"(y), "r"(z), "r"(smem_u32(src))
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // Shared-memory matrix descriptor of a tcgen05 operand in the canonical
@@ -109,12 +136,14 @@ __device__ __forceinline__ void decode_tile(const TcGemmParams& p, int t, int& b
 
 template <bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcGemmParams p) {
+tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+               const __grid_constant__ CUtensorMap tmOut, const __grid_constant__ CUtensorMap tmU, TcGemmParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kGStages * kABytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kGStages * kBBytes);
+  uint8_t* sE = sB + kGStages * kBBytes;          // epilogue boxes, 1024-byte aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(sE + kEpiBytes);
   uint64_t* empty = full + kGStages;
   uint64_t* acc_full = empty + kGStages;
   uint64_t* acc_empty = acc_full + 2;
@@ -223,8 +252,14 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     if (!ok) atomicExch(&cta_err, 1);
   } else if (warp >= 2) {
     // ---- epilogue ----------------------------------------------------------
+    // Warp q drains TMEM lanes 32q..32q+31 (tile rows), 32 columns at a time,
+    // into a 32 x 32 box of shared memory laid out as the 128-byte-swizzled
+    // TMA box (16-byte chunk j of row r at chunk j ^ (r & 7)), then lane 0
+    // stores it.  Two boxes per warp alternate; a box is rewritten only after
+    // the bulk group that read it has finished reading.
     const int q = warp & 3;              // TMEM lane quarter this warp may read
-    const int row_in_tile = q * 32 + lane;
+    uint8_t* box0 = sE + (size_t)(warp - 2) * 2 * kStageBox;
+    int nbox = 0;
     for (int i = 0; i < my_tiles; ++i) {
       int b, mt, nt;
       decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
@@ -234,38 +269,46 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         break;
       }
       tc_fence_after();
-      const int m = mt * kTM + row_in_tile;
-      const bool mvalid = m < p.m_valid[b];
+      const int row0 = mt * kTM + q * 32;              // first tile row of this warp
+      const bool rows_exist = !p.backward || row0 < p.m_limit;
+      const float sc = p.backward ? p.scale[b] : 1.0f;
       const uint32_t t_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTN);
       for (int ch = 0; ch < kTN / 32; ++ch) {
         uint32_t r[32];
         tmem_ld32(t_base + ch * 32, r);
         tmem_ld_wait();
-        const int n0 = nt * kTN + ch * 32;
-        if (!mvalid || n0 >= p.n_valid) continue;
-        if (!p.backward) {
-          float4* dst = reinterpret_cast<float4*>(p.out + (p.out_row0[b] + m) * p.out_ld + n0);
+        if (!rows_exist) continue;
+        uint8_t* box = box0 + (nbox & 1) * kStageBox;
+        if (lane == 0 && nbox >= 2) bulk_wait_read1();
+        __syncwarp();
+        float4* rowp = reinterpret_cast<float4*>(box + lane * 128);
 #pragma unroll
-          for (int v = 0; v < 8; ++v)
-            dst[v] = make_float4(__uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1]),
-                                 __uint_as_float(r[4 * v + 2]), __uint_as_float(r[4 * v + 3]));
-        } else {
-          const float sc = p.scale[b];
-          for (int k = 0; k < p.ndest; ++k) {
-            const int dd = p.dest[(int64_t)b * p.ndest + k];
-            if (dd < 0) continue;
-            float4* dst = reinterpret_cast<float4*>(p.out + (int64_t)dd * p.dest_stride + (int64_t)m * p.out_ld + n0);
-#pragma unroll
-            for (int v = 0; v < 8; ++v)
-              dst[v] = make_float4(sc * __uint_as_float(r[4 * v]), sc * __uint_as_float(r[4 * v + 1]),
-                                   sc * __uint_as_float(r[4 * v + 2]), sc * __uint_as_float(r[4 * v + 3]));
+        for (int v = 0; v < 8; ++v)
+          rowp[v ^ (lane & 7)] = make_float4(sc * __uint_as_float(r[4 * v]), sc * __uint_as_float(r[4 * v + 1]),
+                                             sc * __uint_as_float(r[4 * v + 2]), sc * __uint_as_float(r[4 * v + 3]));
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          const int n0 = nt * kTN + ch * 32;
+          if (!p.backward) {
+            tma_store_2d(&tmOut, box, n0, (int)p.out_row0[b] + row0);
+          } else {
+            for (int k = 0; k < p.ndest; ++k) {
+              const int dd = p.dest[(int64_t)b * p.ndest + k];
+              if (dd >= 0) tma_store_3d(&tmOut, box, n0, row0, dd);
+            }
+            if (p.u_reduce) tma_reduce_add_3d(&tmU, box, n0, row0, p.u_slot);
           }
+          bulk_commit();
         }
+        ++nbox;
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[acc]);
     }
+    if (lane == 0) bulk_wait_all();      // stores done before the CTA exits
+    __syncwarp();
   }
   __syncthreads();
   if (warp == 1) {
@@ -316,12 +359,27 @@ bool make_tmap_bf16(void* tm_out, const void* base, uint64_t inner, uint64_t out
   return r == CUDA_SUCCESS;
 }
 
+bool make_tmap_f32_box32(void* tm_out, const void* base, int rank, const uint64_t* dims, const uint64_t* strides) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn || rank < 2 || rank > 3) return false;
+  cuuint64_t d[3], st[2];
+  cuuint32_t box[3] = {32, 32, 1}, estr[3] = {1, 1, 1};
+  for (int i = 0; i < rank; ++i) d[i] = dims[i];
+  for (int i = 0; i < rank - 1; ++i) st[i] = strides[i];
+  const CUresult r = fn(reinterpret_cast<CUtensorMap*>(tm_out), CU_TENSOR_MAP_DATA_TYPE_FLOAT32, (cuuint32_t)rank,
+                        const_cast<void*>(base), d, st, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 static size_t gemm_smem_bytes() {
-  return 1024 + kGStages * (size_t)(kABytes + kBBytes) + sizeof(uint64_t) * (2 * kGStages + 4) + 16;
+  return 1024 + kGStages * (size_t)(kABytes + kBBytes) + kEpiBytes + sizeof(uint64_t) * (2 * kGStages + 4) + 16;
 }
 
 template <bool A_MN, bool B_MN>
-static cudaError_t launch_tc(const void* tmA, const void* tmB, const TcGemmParams& p, int grid, cudaStream_t st) {
+static cudaError_t launch_tc(const void* tmA, const void* tmB, const void* tmOut, const void* tmU,
+                             const TcGemmParams& p, int grid, cudaStream_t st) {
   auto kern = tc_gemm_kernel<A_MN, B_MN>;
   const size_t smem = gemm_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -336,18 +394,21 @@ static cudaError_t launch_tc(const void* tmA, const void* tmB, const TcGemmParam
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.pdl ? 1 : 0;
-  CUtensorMap a, b;
+  CUtensorMap a, b, o, u;
   std::memcpy(&a, tmA, sizeof(CUtensorMap));
   std::memcpy(&b, tmB, sizeof(CUtensorMap));
-  return cudaLaunchKernelEx(&cfg, kern, a, b, p);
+  std::memcpy(&o, tmOut, sizeof(CUtensorMap));
+  std::memcpy(&u, tmU ? tmU : tmOut, sizeof(CUtensorMap));
+  return cudaLaunchKernelEx(&cfg, kern, a, b, o, u, p);
 }
 
-cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const TcGemmParams& p, bool a_mn, bool b_mn, int grid,
-                           cudaStream_t st) {
+cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, const void* tmU, const TcGemmParams& p,
+                           bool a_mn, bool b_mn, int grid, cudaStream_t st) {
   if (p.total_tiles <= 0) return cudaSuccess;
+  if (p.u_reduce && !tmU) return cudaErrorInvalidValue;
   if (grid > p.total_tiles) grid = p.total_tiles;
-  if (!a_mn && !b_mn) return launch_tc<false, false>(tmA, tmB, p, grid, st);
-  if (a_mn && b_mn) return launch_tc<true, true>(tmA, tmB, p, grid, st);
+  if (!a_mn && !b_mn) return launch_tc<false, false>(tmA, tmB, tmOut, tmU, p, grid, st);
+  if (a_mn && b_mn) return launch_tc<true, true>(tmA, tmB, tmOut, tmU, p, grid, st);
   return cudaErrorInvalidValue;
 }
 
