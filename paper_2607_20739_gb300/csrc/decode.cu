@@ -82,8 +82,76 @@ __global__ void __launch_bounds__(kDecX * kDecY) decode_kernel(DecodeArgs a) {
   decode_chunks(a, pl, red, (int)threadIdx.x, blockIdx.x, gridDim.x, bar);
 }
 
+// Sum of cnt float4 loads base[off(j)], j = 0..cnt-1, issued eight at a time
+// so that each thread keeps eight independent loads in flight.
+template <class Off>
+__device__ __forceinline__ float4 sum_loads8(const float4* base, int cnt, Off off) {
+  float4 acc = f4zero();
+  for (int j0 = 0; j0 < cnt; j0 += 8) {
+    float4 v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = j0 + j < cnt ? __ldcg(base + off(j0 + j)) : f4zero();
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc = f4add(acc, v[j]);
+  }
+  return acc;
+}
+
+// Decode + SGD for large P: one thread per float4 column, grid-stride, no
+// barriers after the plan.  Same arithmetic as decode_chunks.
+__global__ void __launch_bounds__(256) decode_wide_kernel(DecodeArgs a) {
+  __shared__ DecodePlan pl;
+  grid_dep_launch();
+  if (threadIdx.x < 32) derive_plan_warp(a, pl, threadIdx.x);   // needs only the mask
+  __syncthreads();
+  grid_dep_wait();
+  if (blockIdx.x == 0 && threadIdx.x < 32) write_coeffs_warp(a, threadIdx.x);
+  const int64_t P4 = a.P / 4;
+  const int c = a.c;
+  const float4* store = reinterpret_cast<const float4*>(a.store);
+  float4* U = reinterpret_cast<float4*>(a.U);
+  const int64_t slotP = (int64_t)c * P4;           // float4s per store
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P4; p += (int64_t)gridDim.x * blockDim.x) {
+    float4 V = f4zero();
+    if (a.slot < 0) {
+      for (int o = 0; o < c; ++o) {
+        const float4 u = sum_loads8(store + (int64_t)o * P4 + p, a.owners, [&](int r) { return (int64_t)r * slotP; });
+        U[(int64_t)o * P4 + p] = u;
+        V = f4add(V, u);
+      }
+    } else {
+      const int skip = a.u_ready ? -1 : a.slot;      // the slot re-summed below
+      const int nu = a.u_ready ? c : c - 1;
+      V = sum_loads8(U + p, nu, [&](int j) { return (int64_t)(skip >= 0 && j >= skip ? j + 1 : j) * P4; });
+      if (!a.u_ready) {
+        const float4 u =
+            sum_loads8(store + (int64_t)a.slot * P4 + p, a.owners, [&](int r) { return (int64_t)r * slotP; });
+        U[(int64_t)a.slot * P4 + p] = u;
+        V = f4add(V, u);
+      }
+    }
+    float4 D = f4zero();
+    for (int q = 0; q < pl.ndev; ++q) {
+      const float4 Cr = sum_loads8(store + (int64_t)pl.dev[q] * slotP + p, c, [&](int o) { return (int64_t)o * P4; });
+      D = f4fma(pl.devc[q], Cr, D);
+    }
+    const float4 g = f4fma(pl.B, V, D);
+    float4 w = __ldcg(reinterpret_cast<const float4*>(a.w) + p);
+    w = f4fma(-a.lr, g, w);
+    store_outputs(a, p, g, w);
+  }
+}
+
+// Columns from which the one-thread-per-column decode is used.
+constexpr int64_t kWideDecodeMinP4 = 1 << 18;
+
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st, bool pdl, int sm_count) {
   if (a.n > kMaxWorkers || a.owners > kMaxWorkers) return cudaErrorInvalidValue;
+  if (a.P / 4 >= kWideDecodeMinP4) {
+    int64_t blocks = (a.P / 4 + 255) / 256;
+    if (blocks > (int64_t)sm_count * 8) blocks = (int64_t)sm_count * 8;
+    return launch_maybe_pdl(pdl, decode_wide_kernel, dim3((unsigned)blocks), dim3(256), st, a);
+  }
   const int64_t P4 = a.P / 4;
   int64_t chunks = (P4 + kDecX - 1) / kDecX;
   int64_t blocks = chunks < (int64_t)sm_count * 8 ? chunks : (int64_t)sm_count * 8;

@@ -362,7 +362,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   } else {
     // bf16 softmax runs on the tensor cores (PGC_NO_TC=1 keeps the CUDA-core path)
     const char* env = std::getenv("PGC_NO_TC");
-    ctx->tc = dtype == PGC_BF16 && K >= kTcMinClasses && !(env && env[0] == '1');
+    ctx->tc = dtype == PGC_BF16 && K >= kTcMinClasses && K <= kTcMaxClasses && !(env && env[0] == '1');
     ctx->ld = (int64_t)align_up((size_t)d, ctx->tc ? 256 : 64);
     ctx->Ktc = (int64_t)align_up((size_t)K, 256);
   }

@@ -29,6 +29,7 @@ constexpr int kMaxWorkers = 1024;
 // softmax on the tensor cores from this many classes on (the forward N tile is
 // 256 classes; below half a tile the padding outweighs the tensor-core gain)
 constexpr int64_t kTcMinClasses = 128;
+constexpr int64_t kTcMaxClasses = 2048;   // the residual kernel keeps a row in registers
 struct MaskBits {
   uint32_t w[kMaxWorkers / 32];
 };

@@ -147,9 +147,18 @@ __global__ void __launch_bounds__(256) backward_tiled(const T* __restrict__ X, i
 
 // R = softmax(Z) - onehot(y) written as bf16 for the tensor-core backward;
 // one warp per row of an evaluated partition, zero for the padded classes.
-__global__ void softmax_residual_bf16(const float* __restrict__ Z, uint16_t* __restrict__ Rb, int64_t Kpad, int64_t K,
-                                      const int32_t* __restrict__ y, const int64_t* e_row0, const int64_t* e_rows,
-                                      const int64_t* e_zrow0, float* zero_buf, int64_t zero_n4) {
+// R = softmax(Z) - onehot(y) in bf16 for one row per warp, the row held in
+// registers: lane l owns the float4 columns l, l + 32, ... (NV per lane, the
+// padded class count is 128 NV).  Classes K..Kpad-1 and the rows up to the
+// next multiple of 64 (the backward GEMM's K padding) are written as zeros,
+// since another phase may have left values there.  The grid also zeroes
+// zero_buf (the slot total that the backward GEMM accumulates into).
+template <int NV>
+__global__ void __launch_bounds__(256) softmax_residual_bf16(const float* __restrict__ Z, uint16_t* __restrict__ Rb,
+                                                             int64_t K, const int32_t* __restrict__ y,
+                                                             const int64_t* e_row0, const int64_t* e_rows,
+                                                             const int64_t* e_zrow0, float* zero_buf, int64_t zero_n4) {
+  constexpr int64_t Kpad = 128 * NV;
   const int e = blockIdx.y;
   if (zero_buf) {
     const int64_t nthr = (int64_t)gridDim.x * gridDim.y * blockDim.x;
@@ -158,31 +167,54 @@ __global__ void softmax_residual_bf16(const float* __restrict__ Z, uint16_t* __r
   }
   const int lane = threadIdx.x & 31;
   const int64_t rows = e_rows[e];
+  const int64_t rows_pad = (rows + 63) / 64 * 64;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  // rows up to the next multiple of 64 are the backward GEMM's K padding: they
-  // are written as zeros, since another phase may have left values there
-  const int64_t rows_pad = (rows + 63) / 64 * 64;
   for (int64_t r = warp; r < rows_pad; r += nwarps) {
     const int64_t zr = e_zrow0[e] + r;
-    uint16_t* out = Rb + zr * Kpad;
+    uint2* out = reinterpret_cast<uint2*>(Rb + zr * Kpad);
     if (r >= rows) {
-      for (int64_t k = lane; k < Kpad; k += 32) out[k] = 0;
+#pragma unroll
+      for (int j = 0; j < NV; ++j) out[lane + 32 * j] = make_uint2(0u, 0u);
       continue;
     }
-    const float* z = Z + zr * Kpad;
+    const float4* z4 = reinterpret_cast<const float4*>(Z + zr * Kpad);
+    float4 v[NV];
+#pragma unroll
+    for (int j = 0; j < NV; ++j) v[j] = __ldcs(z4 + lane + 32 * j);   // read once: streaming
     float m = -INFINITY;
-    for (int64_t k = lane; k < K; k += 32) m = fmaxf(m, z[k]);
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int64_t k0 = 4 * (lane + 32 * j);
+      if (k0 + 0 < K) m = fmaxf(m, v[j].x);
+      if (k0 + 1 < K) m = fmaxf(m, v[j].y);
+      if (k0 + 2 < K) m = fmaxf(m, v[j].z);
+      if (k0 + 3 < K) m = fmaxf(m, v[j].w);
+    }
     m = warp_max(m);
     float sum = 0.f;
-    for (int64_t k = lane; k < K; k += 32) sum += expf(z[k] - m);
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int64_t k0 = 4 * (lane + 32 * j);
+      v[j].x = k0 + 0 < K ? expf(v[j].x - m) : 0.f;
+      v[j].y = k0 + 1 < K ? expf(v[j].y - m) : 0.f;
+      v[j].z = k0 + 2 < K ? expf(v[j].z - m) : 0.f;
+      v[j].w = k0 + 3 < K ? expf(v[j].w - m) : 0.f;
+      sum += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+    }
     sum = warp_sum(sum);
     const float inv = 1.0f / sum;
     const int lab = y[e_row0[e] + r];
-    for (int64_t k = lane; k < Kpad; k += 32) {
-      const float v = k < K ? expf(z[k] - m) * inv - (k == lab ? 1.0f : 0.0f) : 0.0f;
-      __nv_bfloat16 bv = __float2bfloat16_rn(v);
-      out[k] = *reinterpret_cast<uint16_t*>(&bv);
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int64_t k0 = 4 * (lane + 32 * j);
+      const float r0 = v[j].x * inv - (k0 + 0 == lab ? 1.f : 0.f);
+      const float r1 = v[j].y * inv - (k0 + 1 == lab ? 1.f : 0.f);
+      const float r2 = v[j].z * inv - (k0 + 2 == lab ? 1.f : 0.f);
+      const float r3 = v[j].w * inv - (k0 + 3 == lab ? 1.f : 0.f);
+      __nv_bfloat162 lo = __floats2bfloat162_rn(k0 + 0 < K ? r0 : 0.f, k0 + 1 < K ? r1 : 0.f);
+      __nv_bfloat162 hi = __floats2bfloat162_rn(k0 + 2 < K ? r2 : 0.f, k0 + 3 < K ? r3 : 0.f);
+      out[lane + 32 * j] = make_uint2(*reinterpret_cast<uint32_t*>(&lo), *reinterpret_cast<uint32_t*>(&hi));
     }
   }
 }
@@ -191,10 +223,24 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
                                 const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
                                 int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st) {
   if (nE <= 0) return cudaSuccess;
-  int64_t bx = ((max_rows + 63) / 64 * 64 * 32 + 255) / 256;
-  if (bx > 512) bx = 512;
-  softmax_residual_bf16<<<dim3((unsigned)bx, (unsigned)nE), 256, 0, st>>>(Z, Rb, Kpad, K, y, e_row0, e_rows, e_zrow0,
-                                                                          zero_buf, zero_n / 4);
+  // about four rows per warp, and at least a few CTAs per partition
+  int64_t warps = ((max_rows + 63) / 64 * 64 + 3) / 4;
+  int64_t bx = (warps + 7) / 8;
+  if (bx < 4) bx = 4;
+  if (bx > 1024) bx = 1024;
+  const dim3 grid((unsigned)bx, (unsigned)nE);
+  const int64_t n4 = zero_n / 4;
+  switch (Kpad) {
+    case 256: softmax_residual_bf16<2><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 512: softmax_residual_bf16<4><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 768: softmax_residual_bf16<6><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 1024: softmax_residual_bf16<8><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 1280: softmax_residual_bf16<10><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 1536: softmax_residual_bf16<12><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 1792: softmax_residual_bf16<14><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    case 2048: softmax_residual_bf16<16><<<grid, 256, 0, st>>>(Z, Rb, K, y, e_row0, e_rows, e_zrow0, zero_buf, n4); break;
+    default: return cudaErrorInvalidValue;
+  }
   return cudaGetLastError();
 }
 

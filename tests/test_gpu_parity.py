@@ -40,6 +40,9 @@ CASES = {
     "fr_tc_k256_unequal_rows": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=256, d=600,
                                                                      m=(130, 1, 64, 257)), 5),
     "cr_tc_k128_c_equals_n": (WL["cr_n128_softmax_k1000"].replace(n=3, s=2, K=128, d=256, m=300), 5),
+    # P = K d >= 2^20: the one-thread-per-column decode
+    "cr_tc_wide_decode": (WL["cr_n128_softmax_k1000"].replace(n=5, s=2, K=256, d=4096, m=64), 5),
+    "fr_tc_wide_decode": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=300, d=4000, m=(70, 129, 1, 64)), 5),
 }
 
 
