@@ -44,6 +44,7 @@ struct Phase {
   // tensor-core softmax path: partitions' Z / R rows padded to 64
   std::vector<int64_t> e_zrow0p;
   std::vector<int32_t> f_prefix, f_nk, f_aoff, f_mvalid, b_prefix, b_nk, b_aoff, b_boff, b_mvalid;
+  // f_mvalid / b_mvalid hold the M tiles of each batch (forward: row tiles; backward: class tiles)
   std::vector<int64_t> f_outrow0;
   int64_t zpad_total = 0;
   int64_t* d_e_zrow0p = nullptr;
@@ -115,7 +116,7 @@ struct pgc_ctx {
   int64_t Ktc = 0;           // classes padded to the forward N tile (256)
   uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]
   alignas(64) unsigned char tmXk[128];   // X as K-major A   (box 64 x 128)
-  alignas(64) unsigned char tmW[128];    // Wb as K-major B  (box 64 x 256)
+  alignas(64) unsigned char tmW[128];    // Wb as K-major B  (box 64 x 128: one CTA's half of a 256 tile)
   alignas(64) unsigned char tmR[128];    // R as MN-major A  (box 64 x 64)
   alignas(64) unsigned char tmXm[128];   // X as MN-major B  (box 64 x 64)
   alignas(64) unsigned char tmZo[128];   // Z fp32 output     (box 32 x 32)
@@ -239,13 +240,14 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
         ph.f_nk.push_back((int32_t)(ctx->ld / 64));
         ph.f_aoff.push_back((int32_t)ph.e_row0[e]);
         ph.f_outrow0.push_back(zp);
-        ph.f_mvalid.push_back((int32_t)m);
-        ph.f_prefix.push_back(ph.f_prefix.back() + (int32_t)((m + 127) / 128) * NTf);
+        const int32_t MTf = (int32_t)((m + 127) / 128);
+        ph.f_mvalid.push_back(MTf);
+        ph.f_prefix.push_back(ph.f_prefix.back() + (MTf + 1) / 2 * NTf);   // pairs of row tiles
         ph.b_nk.push_back((int32_t)((m + 63) / 64));
         ph.b_aoff.push_back((int32_t)zp);
         ph.b_boff.push_back((int32_t)ph.e_row0[e]);
-        ph.b_mvalid.push_back((int32_t)ctx->K);
-        ph.b_prefix.push_back(ph.b_prefix.back() + MTb * NTb);
+        ph.b_mvalid.push_back(MTb);
+        ph.b_prefix.push_back(ph.b_prefix.back() + MTb / 2 * NTb);         // pairs of class tiles
         zp += (m + 127) / 128 * 128;   // whole forward tiles: their TMA stores stay inside the partition
       }
       ph.zpad_total = zp;
@@ -520,7 +522,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   if (ctx->tc) {
     const uint64_t pitch = (uint64_t)ctx->ld * 2;
     bool ok = make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, 128) &&
-              make_tmap_bf16(ctx->tmW, ctx->wb, ctx->ld, ctx->Ktc, pitch, 256) &&
+              make_tmap_bf16(ctx->tmW, ctx->wb, ctx->ld, ctx->Ktc, pitch, 128) &&
               make_tmap_bf16(ctx->tmR, ctx->Rb, ctx->Ktc, max_zpad, (uint64_t)ctx->Ktc * 2, 64) &&
               make_tmap_bf16(ctx->tmXm, ctx->X, ctx->ld, ctx->total_rows, pitch, 64);
     const uint64_t zd[2] = {(uint64_t)ctx->Ktc, (uint64_t)max_zpad}, zs[1] = {(uint64_t)ctx->Ktc * 4};
@@ -616,7 +618,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     // G_e = (1/m_e) R_e^T X_e written straight into the stores
     const int nE = (int)ph.parts.size();
     TcGemmParams f = {};
-    f.nbatch = nE; f.tile_prefix = ph.d_f_prefix; f.NT = (int)(ctx->Ktc / 256); f.nk = ph.d_f_nk;
+    f.nbatch = nE; f.tile_prefix = ph.d_f_prefix; f.mt_count = ph.d_f_mvalid; f.NT = (int)(ctx->Ktc / 256); f.nk = ph.d_f_nk;
     // in steady phases every evaluated partition has one store at slot o_t,
     // so the backward also forms U[o_t] = sum_e g_e (TMA reduce-add) and the
     // decode reads it instead of re-summing the stores
@@ -628,7 +630,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
                                     ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows,
                                     u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr, ctx->P, st));
     TcGemmParams b = {};
-    b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
+    b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.mt_count = ph.d_b_mvalid; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
     b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff; b.total_tiles = ph.b_prefix.back(); b.backward = 1;
     b.scale = ph.d_e_scale; b.dest = ph.d_e_dest; b.ndest = ph.ndest; b.m_limit = (int)ctx->K;
     b.u_reduce = u_red ? 1 : 0; b.u_slot = ph.slot;

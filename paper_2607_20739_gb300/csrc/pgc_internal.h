@@ -159,7 +159,8 @@ cudaError_t launch_loss(const LossArgs& a, cudaStream_t st);
 // backward G_e[k][j] = scale_e sum_r R[r][k] X[r][j]  (A = R MN-major, B = X MN-major)
 struct TcGemmParams {
   int nbatch;
-  const int* tile_prefix;   // [nbatch + 1] tiles before batch b (MT_b * NT each)
+  const int* tile_prefix;   // [nbatch + 1] pair tiles before batch b (ceil(MT_b / 2) * NT each)
+  const int* mt_count;      // [nbatch] M tiles (of 128) MT_b
   int NT;                   // N tiles (of 256) per batch
   const int* nk;            // [nbatch] K blocks (of 64)
   const int* a_off;         // [nbatch] A row offset (K-major: M rows; MN-major: K rows)

@@ -5,9 +5,12 @@
 //   backward  G_e[k][j] = (1/m_e) sum_{r in D_e} R[r][k] X[r][j]  A = R (MN-major), B = X (MN-major)
 //
 // with R = softmax(Z) - onehot(y) in bf16 between them.  Both are one
-// persistent, warp-specialised kernel: warp 0 streams 128x64 A tiles and
-// 256x64 B tiles into a 4-stage shared-memory ring with 2-D TMA
-// (cp.async.bulk.tensor, 128-byte swizzle), warp 1 issues
+// persistent, warp-specialised kernel launched as clusters of two CTAs: the
+// pair computes the M tiles 2i and 2i+1 of the same (batch, N tile), so the
+// B tile is common; each CTA loads its own 128x64 A tile and one 128-row half
+// of the 256x64 B tile, multicast into both CTAs, into a 4-stage
+// shared-memory ring with 2-D TMA (cp.async.bulk.tensor, 128-byte swizzle).
+// A stage is refilled once the MMAs of both CTAs have read it.  Warp 1 issues
 // tcgen05.mma.cta_group::1.kind::f16 (bf16 in, fp32 accumulate) into one of
 // two 128x256 TMEM accumulators, and warps 2-5 drain the other accumulator
 // with tcgen05.ld, stage 32 x 32 fp32 boxes in (swizzled) shared memory and
@@ -42,6 +45,24 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* tm, in
           smem_u32(dst)),
       "l"(tm), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* tm, int x, int y, uint64_t* bar,
+                                               uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst)),
+      "l"(tm), "r"(x), "r"(y), "r"(smem_u32(bar)), "h"(mask)
+      : "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, const void* src, int x, int y) {
@@ -101,6 +122,13 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
+// arrive on the barrier at the same offset in every CTA of `mask`
+__device__ __forceinline__ void umma_commit_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+                   smem_u32(bar)),
+               "h"(mask)
+               : "memory");
+}
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -122,7 +150,10 @@ __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.
 // ---------------------------------------------------------------------------
 // the kernel
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void decode_tile(const TcGemmParams& p, int t, int& b, int& mt, int& nt) {
+// Pair tile t -> batch b, N tile nt and this CTA's M tile mt = 2 mp + rank;
+// false when mt is past the batch's M tiles (odd count: the CTA computes a
+// dummy tile to keep the pair in step and stores nothing).
+__device__ __forceinline__ bool decode_tile(const TcGemmParams& p, int t, int rank, int& b, int& mt, int& nt) {
   int lo = 0, hi = p.nbatch - 1;
   while (lo < hi) {                      // last b with tile_prefix[b] <= t
     const int mid = (lo + hi + 1) >> 1;
@@ -130,8 +161,9 @@ __device__ __forceinline__ void decode_tile(const TcGemmParams& p, int t, int& b
   }
   b = lo;
   const int rem = t - p.tile_prefix[b];
-  mt = rem / p.NT;
+  mt = 2 * (rem / p.NT) + rank;
   nt = rem % p.NT;
+  return mt < p.mt_count[b];
 }
 
 template <bool A_MN, bool B_MN>
@@ -151,11 +183,13 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
   __shared__ int cta_err;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rank = (int)cluster_rank();
+  constexpr uint16_t kPair = 0x3;
   if (threadIdx.x == 0) {
     cta_err = 0;
     for (int s = 0; s < kGStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], 2);           // the MMAs of both CTAs read the stage
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&acc_full[a], 1);
@@ -170,16 +204,15 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync_all();                    // the peer's barriers exist before any multicast
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   if (threadIdx.x == 0) grid_dep_launch();
   if (p.pdl) grid_dep_wait();           // inputs are the previous kernels' outputs
 
-  // tiles of this CTA: blockIdx.x, blockIdx.x + gridDim.x, ...
-  const int my_tiles = p.total_tiles > (int)blockIdx.x
-                           ? (p.total_tiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x
-                           : 0;
+  // pair tiles of this cluster: pair, pair + npairs, ...
+  const int pair = (int)blockIdx.x >> 1, npairs = (int)gridDim.x >> 1;
+  const int my_tiles = p.total_tiles > pair ? (p.total_tiles - pair + npairs - 1) / npairs : 0;
 
   if (warp == 0 && lane == 0) {
     // ---- producer ----------------------------------------------------------
@@ -187,10 +220,11 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     bool ok = true;
     for (int i = 0; i < my_tiles && ok; ++i) {
       int b, mt, nt;
-      decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
+      decode_tile(p, pair + i * npairs, rank, b, mt, nt);
       const int nkb = p.nk[b];
       for (int kb = 0; kb < nkb; ++kb, ++it) {
         const int s = it % kGStages;
+        // both CTAs' MMAs are done with the stage (this CTA's B half lands in both)
         if (it >= kGStages && !mbar_wait(&empty[s], ((it / kGStages) - 1) & 1, p.status)) { ok = false; break; }
         mbar_arrive_expect_tx(&full[s], kABytes + kBBytes);
         uint8_t* a_dst = sA + (size_t)s * kABytes;
@@ -202,10 +236,10 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
             tma_load_2d(a_dst + j * 8192, &tmA, mt * kTM + j * 64, p.a_off[b] + kb * kTK, &full[s]);
         }
         if (!B_MN) {
-          tma_load_2d(b_dst, &tmB, kb * kTK, nt * kTN, &full[s]);
+          tma_load_2d_mc(b_dst + rank * (kBBytes / 2), &tmB, kb * kTK, nt * kTN + rank * (kTN / 2), &full[s], kPair);
         } else {
-          for (int j = 0; j < kTN / 64; ++j)
-            tma_load_2d(b_dst + j * 8192, &tmB, nt * kTN + j * 64, p.b_off[b] + kb * kTK, &full[s]);
+          for (int j = 2 * rank; j < 2 * rank + 2; ++j)
+            tma_load_2d_mc(b_dst + j * 8192, &tmB, nt * kTN + j * 64, p.b_off[b] + kb * kTK, &full[s], kPair);
         }
       }
     }
@@ -222,7 +256,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     bool ok = true;
     for (int i = 0; i < my_tiles && ok; ++i) {
       int b, mt, nt;
-      decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
+      decode_tile(p, pair + i * npairs, rank, b, mt, nt);
       const int acc = i & 1;
       if (i >= 2 && !mbar_wait(&acc_empty[acc], ((i / 2) - 1) & 1, p.status)) { ok = false; break; }
       tc_fence_after();
@@ -244,7 +278,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
                                    : smem_desc_sw128(b_base + kk * 32, 16, 1024);
           umma_bf16(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
         }
-        umma_commit(&empty[s]);          // the stage is free once these MMAs finish
+        umma_commit_mc(&empty[s], kPair);  // this CTA is done with the stage, in both CTAs' count
       }
       if (!ok) break;
       umma_commit(&acc_full[acc]);       // the accumulator is complete
@@ -262,7 +296,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     int nbox = 0;
     for (int i = 0; i < my_tiles; ++i) {
       int b, mt, nt;
-      decode_tile(p, blockIdx.x + i * gridDim.x, b, mt, nt);
+      const bool real = decode_tile(p, pair + i * npairs, rank, b, mt, nt);
       const int acc = i & 1;
       if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[acc], (i / 2) & 1, p.status))) {
         atomicExch(&cta_err, 1);
@@ -270,7 +304,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
       tc_fence_after();
       const int row0 = mt * kTM + q * 32;              // first tile row of this warp
-      const bool rows_exist = !p.backward || row0 < p.m_limit;
+      const bool rows_exist = real && (!p.backward || row0 < p.m_limit);
       const float sc = p.backward ? p.scale[b] : 1.0f;
       const uint32_t t_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTN);
       for (int ch = 0; ch < kTN / 32; ++ch) {
@@ -311,6 +345,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     __syncwarp();
   }
   __syncthreads();
+  cluster_sync_all();                    // no multicast or remote arrive is still aimed at this CTA
   if (warp == 1) {
     // every MMA of this CTA has completed before its accumulator was drained;
     // after a failure, wait (bounded) for the last commits before releasing
@@ -389,11 +424,31 @@ static cudaError_t launch_tc(const void* tmA, const void* tmB, const void* tmOut
   cfg.blockDim = dim3(kGemmThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = p.pdl ? 1 : 0;
+  cfg.numAttrs = p.pdl ? 2 : 1;
+  // one pair per two SMs that can hold it at once
+  static int max_pairs[2] = {0, 0};
+  int& mp = max_pairs[A_MN ? 1 : 0];
+  if (mp == 0) {
+    cudaLaunchConfig_t q = cfg;
+    q.gridDim = dim3(2);
+    q.numAttrs = 1;
+    int nc = 0;
+    e = cudaOccupancyMaxActiveClusters(&nc, kern, &q);
+    if (e != cudaSuccess) return e;
+    mp = nc > 0 ? nc : 1;
+  }
+  int pairs = grid / 2 < mp ? grid / 2 : mp;
+  if (pairs > p.total_tiles) pairs = p.total_tiles;
+  if (pairs < 1) pairs = 1;
+  cfg.gridDim = dim3((unsigned)(2 * pairs));
   CUtensorMap a, b, o, u;
   std::memcpy(&a, tmA, sizeof(CUtensorMap));
   std::memcpy(&b, tmB, sizeof(CUtensorMap));
@@ -406,7 +461,6 @@ cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, 
                            bool a_mn, bool b_mn, int grid, cudaStream_t st) {
   if (p.total_tiles <= 0) return cudaSuccess;
   if (p.u_reduce && !tmU) return cudaErrorInvalidValue;
-  if (grid > p.total_tiles) grid = p.total_tiles;
   if (!a_mn && !b_mn) return launch_tc<false, false>(tmA, tmB, tmOut, tmU, p, grid, st);
   if (a_mn && b_mn) return launch_tc<true, true>(tmA, tmB, tmOut, tmU, p, grid, st);
   return cudaErrorInvalidValue;
