@@ -51,6 +51,10 @@ struct Phase {
   int32_t *d_f_prefix = nullptr, *d_f_nk = nullptr, *d_f_aoff = nullptr, *d_f_mvalid = nullptr;
   int32_t *d_b_prefix = nullptr, *d_b_nk = nullptr, *d_b_aoff = nullptr, *d_b_boff = nullptr, *d_b_mvalid = nullptr;
   int64_t* d_f_outrow0 = nullptr;
+  // few-class softmax: 128-row tiles {row0, rows, item, flags} and items
+  std::vector<int32_t> sk_tiles;
+  int sk_items = 0;
+  int32_t* d_sk_tiles = nullptr;
   // device copies
   WorkItem* d_items = nullptr;
   int32_t* d_e_item0 = nullptr;
@@ -113,6 +117,10 @@ struct pgc_ctx {
   bool pdl = true;           // chain the step's kernels with programmatic dependent launch
   int tail_mode = 0;         // fused tail of the gradient kernel (see GradRowsArgs)
   bool tc = false;           // softmax on the tensor cores (bf16 features)
+  bool smallk = false;       // few-class softmax: one-pass cluster kernel
+  int sk_nper = 0;           // its 64-feature blocks per CTA slice
+  int sk_nc = 0;             // its clusters
+  alignas(64) unsigned char tmW16[128];  // Wb [16][ld] for the few-class kernel (box 64 x 16)
   int64_t Ktc = 0;           // classes padded to the forward N tile (256)
   uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]
   alignas(64) unsigned char tmXk[128];   // X as K-major A   (box 64 x 128)
@@ -227,6 +235,34 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
       }
       ph.e_item0.push_back((int32_t)ph.items.size());
     }
+  } else if (ctx->smallk) {
+    // 128-row tiles in partition order; cluster c takes [T c / nc, T (c+1) / nc);
+    // one item per cluster and partition it touches
+    std::vector<int32_t> te;              // partition of each tile
+    for (int e = 0; e < nE; ++e)
+      for (int64_t r0 = 0; r0 < ph.e_rows[e]; r0 += 128) {
+        ph.sk_tiles.push_back((int32_t)(ph.e_row0[e] + r0));
+        ph.sk_tiles.push_back((int32_t)std::min<int64_t>(128, ph.e_rows[e] - r0));
+        ph.sk_tiles.push_back(0);
+        ph.sk_tiles.push_back(0);
+        te.push_back(e);
+      }
+    const int64_t T = (int64_t)te.size(), nc = ctx->sk_nc;
+    std::vector<int32_t> items_of(nE, 0);
+    int item = 0;
+    for (int64_t cl = 0; cl < nc; ++cl) {
+      const int64_t a = T * cl / nc, b = T * (cl + 1) / nc;
+      for (int64_t i = a; i < b; ++i) {
+        const bool first = i == a || te[i] != te[i - 1];
+        const bool last = i == b - 1 || te[i] != te[i + 1];
+        if (first) { ++items_of[te[i]]; ++item; }
+        ph.sk_tiles[4 * i + 2] = item - 1;
+        ph.sk_tiles[4 * i + 3] = (first ? 1 : 0) | (last ? 2 : 0);
+      }
+    }
+    ph.sk_items = item;
+    ph.e_item0.push_back(0);
+    for (int e = 0; e < nE; ++e) ph.e_item0.push_back(ph.e_item0.back() + items_of[e]);
   } else {
     for (int e = 0; e <= nE; ++e) ph.e_item0.push_back(e);
     if (ctx->tc) {
@@ -367,6 +403,12 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
     ctx->tc = dtype == PGC_BF16 && K >= kTcMinClasses && K <= kTcMaxClasses && !(env && env[0] == '1');
     ctx->ld = (int64_t)align_up((size_t)d, ctx->tc ? 256 : 64);
     ctx->Ktc = (int64_t)align_up((size_t)K, 256);
+    const char* env2 = std::getenv("PGC_NO_SMALLK");
+    if (!ctx->tc && dtype == PGC_BF16 && !(env2 && env2[0] == '1') && smallk_fits(K, ctx->ld)) {
+      ctx->sk_nper = (int)((ctx->ld / 64 + 7) / 8);
+      ctx->sk_nc = smallk_max_clusters(ctx->sk_nper);
+      ctx->smallk = ctx->sk_nc > 0;
+    }
   }
   ctx->P = ctx->K * ctx->ld;
   ctx->Kpad = (int64_t)align_up((size_t)K, 4);
@@ -396,6 +438,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   for (auto& ph : ctx->phases) {
     // the tensor-core backward writes the stores directly: no partials
     const size_t np = ctx->tc ? 0
+                      : ctx->smallk ? (size_t)ph.sk_items * ctx->P
                       : ctx->loss == PGC_SOFTMAX ? ph.parts.size() * (size_t)ctx->P
                                                  : ph.items.size() * (size_t)ctx->ld;
     max_partials = std::max(max_partials, np);
@@ -404,7 +447,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   std::vector<uint8_t> tab;
   size_t off = 0;
   std::vector<size_t> offs;
-  constexpr int kTabs = 18;
+  constexpr int kTabs = 19;
   for (auto& ph : ctx->phases) {
     offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
@@ -424,6 +467,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_aoff);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_boff);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_mvalid);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.sk_tiles);
   }
   // loss chunks (softmax): {row0, rows, 0} per chunk
   std::vector<int64_t> ldesc;
@@ -454,7 +498,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   PGC_ALLOC(ctx->X, (size_t)ctx->total_rows * ctx->ld * ctx->esize);
   PGC_ALLOC(ctx->y, (size_t)ctx->total_rows * 4 + 64);   // per-stage label copies overrun by <= 12 B
   PGC_ALLOC(ctx->w, Pb);
-  const size_t wb_elems = ctx->tc ? (size_t)ctx->Ktc * ctx->ld : (size_t)ctx->P;
+  const size_t wb_elems = ctx->tc ? (size_t)ctx->Ktc * ctx->ld : ctx->smallk ? (size_t)16 * ctx->ld : (size_t)ctx->P;
   if (dtype == PGC_BF16) PGC_ALLOC(ctx->wb, wb_elems * 2);
   PGC_ALLOC(ctx->store, (size_t)ctx->owners * ctx->c * Pb);
   PGC_ALLOC(ctx->U, (size_t)ctx->c * Pb);
@@ -516,9 +560,16 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
     ph.d_b_aoff = reinterpret_cast<int32_t*>(base + o[15]);
     ph.d_b_boff = reinterpret_cast<int32_t*>(base + o[16]);
     ph.d_b_mvalid = reinterpret_cast<int32_t*>(base + o[17]);
+    ph.d_sk_tiles = reinterpret_cast<int32_t*>(base + o[18]);
   }
   ctx->loss_desc = nullptr;
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
+  if (ctx->smallk) {
+    const uint64_t pitch = (uint64_t)ctx->ld * 2;
+    if (!make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, 128) ||
+        !make_tmap_bf16(ctx->tmW16, ctx->wb, ctx->ld, 16, pitch, 16))
+      return fail(cudaErrorInvalidValue);
+  }
   if (ctx->tc) {
     const uint64_t pitch = (uint64_t)ctx->ld * 2;
     bool ok = make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, 128) &&
@@ -639,6 +690,14 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     dc.u_ready = u_red ? 1 : 0;
     nl[PGC_KGRAD] = 3;
     need_commit = false;
+  } else if (ctx->smallk) {
+    SmallKArgs a;
+    a.tiles = reinterpret_cast<const int4*>(ph.d_sk_tiles); a.ntiles = (int)(ph.sk_tiles.size() / 4);
+    a.nkb = (int)(ctx->ld / 64); a.nper = ctx->sk_nper; a.K = (int)ctx->K;
+    a.y = static_cast<const int32_t*>(ctx->y); a.partials = ctx->partials; a.P = ctx->P; a.ld = ctx->ld;
+    a.status = ctx->status; a.pdl = ctx->pdl ? 1 : 0;
+    nl[PGC_KGRAD] = 1;
+    PGC_CK(ctx, launch_softmax_smallk(ctx->tmXk, ctx->tmW16, a, ctx->sk_nc, st));
   } else {
     SoftmaxCCArgs a;
     a.dtype = ctx->dtype; a.ld = ctx->ld; a.K = ctx->K; a.X = ctx->X; a.y = static_cast<const int32_t*>(ctx->y);

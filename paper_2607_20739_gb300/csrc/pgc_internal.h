@@ -198,6 +198,29 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
                                 const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
                                 int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st);
 
+// ---- softmax with few classes: one pass over X per step --------------------
+// tiles[i] = {first global X row, rows (<= 128), item, flags: 1 first / 2 last
+// tile of a cluster's run in one partition}; cluster c of nc takes tiles
+// [ntiles c / nc, ntiles (c + 1) / nc).  partials[item][K][ld] receives the
+// unscaled gradient sums of the run.
+struct SmallKArgs {
+  const int4* tiles;
+  int ntiles;
+  int nkb;                  // ld / 64
+  int nper;                 // 64-feature blocks per CTA slice (ceil(nkb / 8))
+  int K;
+  const int32_t* y;         // labels per global row
+  float* partials;
+  int64_t P;                // K * ld
+  int64_t ld;
+  int* status;
+  int pdl;
+};
+bool smallk_fits(int64_t K, int64_t ld);
+int smallk_max_clusters(int nper);
+cudaError_t launch_softmax_smallk(const void* tmX, const void* tmW, const SmallKArgs& a, int nclusters,
+                                  cudaStream_t st);
+
 // ---- misc -------------------------------------------------------------------
 cudaError_t launch_f32_to_bf16(const float* src, uint16_t* dst, int64_t count, cudaStream_t st);
 

@@ -40,6 +40,11 @@ CASES = {
     "fr_tc_k256_unequal_rows": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=256, d=600,
                                                                      m=(130, 1, 64, 257)), 5),
     "cr_tc_k128_c_equals_n": (WL["cr_n128_softmax_k1000"].replace(n=3, s=2, K=128, d=256, m=300), 5),
+    # few-class softmax (one-pass cluster kernel): ragged tiles, partition
+    # boundaries inside a cluster's run, empty feature slices, K = 16
+    "fr_smallk_k10_unequal_rows": (WL["fr_n32_softmax_k10"].replace(n=4, s=1, d=3072, m=(300, 1, 129, 700)), 5),
+    "cr_smallk_k16_d1000": (WL["fr_n32_softmax_k10"].replace(scheme="CR", n=6, s=2, K=16, d=1000, m=257), 5),
+    "cr_smallk_k5_d64": (WL["fr_n32_softmax_k10"].replace(scheme="CR", n=5, s=1, K=5, d=64, m=(1, 2, 128, 129, 40)), 5),
     # P = K d >= 2^20: the one-thread-per-column decode
     "cr_tc_wide_decode": (WL["cr_n128_softmax_k1000"].replace(n=5, s=2, K=256, d=4096, m=64), 5),
     "fr_tc_wide_decode": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=300, d=4000, m=(70, 129, 1, 64)), 5),
