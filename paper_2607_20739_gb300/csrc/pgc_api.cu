@@ -236,13 +236,13 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
       ph.e_item0.push_back((int32_t)ph.items.size());
     }
   } else if (ctx->smallk) {
-    // 128-row tiles in partition order; cluster c takes [T c / nc, T (c+1) / nc);
+    // kSmallKRows-row tiles in partition order; cluster c takes [T c / nc, T (c+1) / nc);
     // one item per cluster and partition it touches
     std::vector<int32_t> te;              // partition of each tile
     for (int e = 0; e < nE; ++e)
-      for (int64_t r0 = 0; r0 < ph.e_rows[e]; r0 += 128) {
+      for (int64_t r0 = 0; r0 < ph.e_rows[e]; r0 += kSmallKRows) {
         ph.sk_tiles.push_back((int32_t)(ph.e_row0[e] + r0));
-        ph.sk_tiles.push_back((int32_t)std::min<int64_t>(128, ph.e_rows[e] - r0));
+        ph.sk_tiles.push_back((int32_t)std::min<int64_t>(kSmallKRows, ph.e_rows[e] - r0));
         ph.sk_tiles.push_back(0);
         ph.sk_tiles.push_back(0);
         te.push_back(e);
@@ -566,7 +566,7 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
   if (ctx->smallk) {
     const uint64_t pitch = (uint64_t)ctx->ld * 2;
-    if (!make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, 128) ||
+    if (!make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, kSmallKRows) ||
         !make_tmap_bf16(ctx->tmW16, ctx->wb, ctx->ld, 16, pitch, 16))
       return fail(cudaErrorInvalidValue);
   }

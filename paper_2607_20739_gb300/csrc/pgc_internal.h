@@ -199,10 +199,11 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
                                 int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st);
 
 // ---- softmax with few classes: one pass over X per step --------------------
-// tiles[i] = {first global X row, rows (<= 128), item, flags: 1 first / 2 last
+// tiles[i] = {first global X row, rows (<= kSmallKRows), item, flags: 1 first / 2 last
 // tile of a cluster's run in one partition}; cluster c of nc takes tiles
 // [ntiles c / nc, ntiles (c + 1) / nc).  partials[item][K][ld] receives the
 // unscaled gradient sums of the run.
+constexpr int kSmallKRows = 128;    // rows per tile of the few-class kernel
 struct SmallKArgs {
   const int4* tiles;
   int ntiles;

@@ -38,7 +38,9 @@ namespace pgc {
 namespace {
 
 constexpr int kCS = 8;                 // CTAs per cluster (feature slices)
-constexpr int kRows = 128;             // rows per tile (MMA M of the forward)
+constexpr int kRows = kSmallKRows;     // rows per tile (MMA M of the forward)
+static_assert(kRows == 128, "the forward accumulator layout assumes M = 128");
+constexpr int kTileCache = 128;        // tile descriptors kept in shared memory
 constexpr int kNC = 16;                // padded classes (MMA N)
 constexpr int kThreads = 192;          // producer, MMA, 4 epilogue warps
 constexpr uint32_t kBox = kRows * 64 * 2;      // one 128 x 64 bf16 X box
@@ -137,6 +139,10 @@ __device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t
       "l"(a), "l"(b), "r"(id), "r"(acc)
       : "memory");
 }
+// accumulate into D (no predicate computation on the issue path)
+__device__ __forceinline__ void mma_acc(uint32_t d, uint64_t a, uint64_t b, uint32_t id) {
+  asm volatile("tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, 1;" ::"r"(d), "l"(a), "l"(b), "r"(id) : "memory");
+}
 __device__ __forceinline__ void commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
@@ -169,7 +175,7 @@ __device__ __forceinline__ uint32_t r_offset(int k, int r) {
 
 // Shared-memory plan; offsets from the 1024-byte aligned base.
 struct SkSmem {
-  uint32_t slots, slot_bytes, wsm, zred, rstage, rbuf, bars, total;
+  uint32_t slots, slot_bytes, wsm, zred, rstage, rbuf, tiles, bars, total;
 };
 __host__ __device__ static SkSmem sk_smem(int nper) {
   SkSmem s;
@@ -180,7 +186,8 @@ __host__ __device__ static SkSmem sk_smem(int nper) {
   s.zred = s.wsm + (uint32_t)((nper * kWBox + 1023) & ~1023);
   s.rstage = s.zred + kCS * kZPart;
   s.rbuf = s.rstage + 2 * kRBlock;
-  s.bars = s.rbuf + 2 * kCS * kRBlock;
+  s.tiles = s.rbuf + 2 * kCS * kRBlock;
+  s.bars = s.tiles + kTileCache * 16;
   s.total = s.bars + 32 * 8 + 16;
   return s;
 }
@@ -207,6 +214,7 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
   uint64_t* gempty = bars + 14;      // [2]
   uint64_t* mma_done = bars + 16;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
+  int4* tcache = reinterpret_cast<int4*>(sm + L.tiles);  // this cluster's first tile descriptors
   __shared__ int cta_err;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -220,6 +228,8 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
   const int t0 = (int)((int64_t)a.ntiles * cid / ncl), t1 = (int)((int64_t)a.ntiles * (cid + 1) / ncl);
   const int n = t1 - t0;
 
+  for (int i = threadIdx.x; i < n && i < kTileCache; i += blockDim.x) tcache[i] = a.tiles[t0 + i];
+  auto tile_desc = [&](int i) { return i < kTileCache ? tcache[i] : a.tiles[t0 + i]; };
   if (threadIdx.x == 0) {
     cta_err = 0;
     for (int i = 0; i < 2; ++i) {
@@ -264,7 +274,7 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
     int issued = 0;
     auto load_x = [&](int i) {
       const int s = i & 1;
-      const int4 tl = a.tiles[t0 + i];
+      const int4 tl = tile_desc(i);
       mbar_arrive_expect_tx(&slot_full[s], (uint32_t)nk * kBox);
       for (int j = 0; j < nk; ++j)
         tma_load_2d(slot0 + s * L.slot_bytes + j * kBox, &tmX, (kb0 + j) * 64, tl.x, &slot_full[s]);
@@ -288,44 +298,73 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
     }
     mbar_wait(wfull, 0, a.status);
   } else if (warp == 1 && lane == 0) {
-    // ---- MMA issuer: fwd(0), fwd(1), bwd(0), fwd(2), bwd(1), ... -----------
+    // ---- MMA issuer ----------------------------------------------------------
+    // Forward of tile f once its X slice landed (at most two tiles ahead of
+    // the backward: two X slots); backward of tile b as soon as its R block
+    // arrived.  Whichever is ready goes first, so a slot is released as soon
+    // as its exchange completes.  Readiness is probed with test_wait, which
+    // never suspends the thread; descriptors are formed once per operand and
+    // stepped by constants (the address field counts 16-byte units).
     constexpr uint32_t id_fwd = idesc(kRows, kNC, false, false);
     constexpr uint32_t id_bwd = idesc(kRows, kNC, true, false);
     bool ok = mbar_wait(wfull, 0, a.status);
-    int seg = -1;
-    for (int i = 0; i <= n && ok; ++i) {
-      if (i < n) {
-        const int s = i & 1;
-        if (!mbar_wait(&slot_full[s], (i >> 1) & 1, a.status)) { ok = false; break; }
-        if (i >= 2 && !mbar_wait(&zacc_empty[s], ((i >> 1) - 1) & 1, a.status)) { ok = false; break; }
-        fence_after();
-        const uint32_t base = smem_u32(slot0 + s * L.slot_bytes);
-        for (int j = 0; j < nk; ++j)
+    int seg = -1, f = 0, b = 0;
+    uint64_t t_idle = 0;
+    uint32_t spins = 0;
+    while (ok && b < n) {
+      bool did = false;
+      if (b < f && mbar_test_wait(&rfull[b & 1], (b >> 1) & 1)) {
+        const int s = b & 1;
+        const int4 tl = tile_desc(b);
+        const bool first = (tl.w & 1) || b == 0, last = (tl.w & 2) || b == n - 1;
+        const int g = (seg + (first ? 1 : 0)) & 1;
+        if (!first || seg + 1 < 2 || mbar_test_wait(&gempty[g], (((seg + 1) >> 1) - 1) & 1)) {
+          if (first) ++seg;
+          if (b + 2 < n) mbar_arrive_expect_tx(&rfull[s], kCS * kRBlock);
+          fence_after();
+          const uint32_t base = smem_u32(slot0 + s * L.slot_bytes);
+          const uint64_t db = sdesc(smem_u32(rbuf + s * kCS * kRBlock), 256, 128, 0);
+          for (int mt = 0; mt < nmt; ++mt) {
+            const uint64_t da = sdesc(base + 2 * mt * kBox, kBox, 1024, 2);
+            const uint32_t d = tmem + gacc_col(g) + mt * kNC;
+            mma(d, da, db, id_bwd, first ? 0u : 1u);
 #pragma unroll
-          for (int kk = 0; kk < 4; ++kk)
-            mma(tmem + zacc_col(s), sdesc(base + j * kBox + kk * 32, 16, 1024, 2),
-                sdesc(smem_u32(wsm) + j * kWBox + kk * 32, 16, 1024, 2), id_fwd, (j | kk) != 0 ? 1u : 0u);
-        commit(&zacc_full[s]);
+            for (int kk = 1; kk < kRows / 16; ++kk) mma_acc(d, da + kk * 128, db + kk * 32, id_bwd);
+          }
+          commit(&slot_empty[s]);
+          if (last) commit(&gfull[g]);
+          ++b;
+          did = true;
+        }
       }
-      if (i >= 1) {
-        const int ib = i - 1, s = ib & 1;
-        const int4 tl = a.tiles[t0 + ib];
-        const bool first = (tl.w & 1) || ib == 0, last = (tl.w & 2) || ib == n - 1;
-        if (first) ++seg;
-        const int g = seg & 1;
-        if (!mbar_wait(&rfull[s], (ib >> 1) & 1, a.status)) { ok = false; break; }
-        if (ib + 2 < n) mbar_arrive_expect_tx(&rfull[s], kCS * kRBlock);
-        if (first && seg >= 2 && !mbar_wait(&gempty[g], ((seg >> 1) - 1) & 1, a.status)) { ok = false; break; }
+      if (!did && f < n && f - b < 2 && mbar_test_wait(&slot_full[f & 1], (f >> 1) & 1) &&
+          (f < 2 || mbar_test_wait(&zacc_empty[f & 1], ((f >> 1) - 1) & 1))) {
+        const int s = f & 1;
         fence_after();
-        const uint32_t base = smem_u32(slot0 + s * L.slot_bytes);
-        const uint32_t rb = smem_u32(rbuf + s * kCS * kRBlock);
-        for (int mt = 0; mt < nmt; ++mt)
-#pragma unroll
-          for (int kk = 0; kk < kRows / 16; ++kk)
-            mma(tmem + gacc_col(g) + mt * kNC, sdesc(base + 2 * mt * kBox + kk * 2048, kBox, 1024, 2),
-                sdesc(rb + kk * 512, 256, 128, 0), id_bwd, (first && kk == 0) ? 0u : 1u);
-        commit(&slot_empty[s]);
-        if (last) commit(&gfull[g]);
+        const uint64_t da0 = sdesc(smem_u32(slot0 + s * L.slot_bytes), 16, 1024, 2);
+        const uint64_t db0 = sdesc(smem_u32(wsm), 16, 1024, 2);
+        const uint32_t d = tmem + zacc_col(s);
+        for (int j = 0; j < nk; ++j) {
+          const uint64_t da = da0 + j * (kBox >> 4), db = db0 + j * (kWBox >> 4);
+          mma(d, da, db, id_fwd, j != 0 ? 1u : 0u);
+          mma_acc(d, da + 2, db + 2, id_fwd);
+          mma_acc(d, da + 4, db + 4, id_fwd);
+          mma_acc(d, da + 6, db + 6, id_fwd);
+        }
+        commit(&zacc_full[s]);
+        ++f;
+        did = true;
+      }
+      if (did) {
+        t_idle = 0;
+        spins = 0;
+      } else {
+        // bounded like every other wait: give up after kWaitMaxNs without progress
+        if (t_idle == 0) t_idle = globaltimer_ns();
+        if (++spins > kWaitMaxIters || ((spins & 63u) == 0 && globaltimer_ns() - t_idle > kWaitMaxNs)) {
+          atomicOr(a.status, kErrWaitTimeout);
+          ok = false;
+        }
       }
     }
     if (!ok) atomicExch(&cta_err, 1);
@@ -343,7 +382,7 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
     bool waited = false;
     for (int i = 0; i < n && ok; ++i) {
       const int s = i & 1;
-      const int4 tl = a.tiles[t0 + i];
+      const int4 tl = tile_desc(i);
       const bool first = (tl.w & 1) || i == 0, last = (tl.w & 2) || i == n - 1;
       if (first) ++seg;
       // (1) drain this CTA's partial Z of the tile
