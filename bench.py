@@ -39,7 +39,6 @@ from paper_2607_20739_gb300 import workloads as W  # noqa: E402
 METRIC = "PGC steps/s & samples/s at 1 GB300; % of HBM (or bf16 TC) roofline"
 DEFAULT_WORKLOAD = "cr_n8_logistic_d1024"
 L2_BYTES = 129 * 2 ** 20
-KERNEL_NAMES = ["gradient", "commit", "decode"]
 
 
 def parse_args(argv=None):
@@ -88,13 +87,36 @@ def grad_bytes_per_row(w: W.Workload) -> int:
     return w.d * esz + 4
 
 
+TC_MIN_CLASSES = 128          # the library runs bf16 softmax from this many classes on the tensor cores
+
+
+def tensor_core_path(w: W.Workload) -> bool:
+    return w.loss == "softmax" and w.dtype == "bf16" and TC_MIN_CLASSES <= w.K <= 2048
+
+
 def roofline_model(w: W.Workload, peaks: dict):
-    """(bound, algorithmic units per gradient launch, unit name, peak)."""
+    """(bound, algorithmic units per launch of the dominant kernel, unit, peak).
+
+    Streaming paths: the gradient kernel reads the evaluated partitions' X and
+    labels once (bytes).  Tensor-core softmax: each of the two GEMMs (logits
+    X W^T and gradient R^T X) performs 2 rows d K flops per step; the slower
+    of the two is reported."""
     rows = evaluated_rows(w)
-    if w.loss == "softmax" and w.K >= 256:
-        flops = 2.0 * 2.0 * rows * w.d * w.K
+    if tensor_core_path(w):
+        flops = 2.0 * rows * w.d * w.K
         return "tensor", flops, "TFLOP/s", peaks.get("bf16_tflops_sustained") or 1700.0
     return "hbm", float(rows * grad_bytes_per_row(w)), "GB/s", peaks.get("hbm_gbs") or 6800.0
+
+
+def kernel_label(w: W.Workload, single: bool, dom: int) -> str:
+    if tensor_core_path(w):
+        return ("tc_gemm_kernel, gradient R^T X" if dom == 2 else "tc_gemm_kernel, logits X W^T") + \
+            " (tcgen05, 2-CTA clusters)"
+    if w.loss == "softmax" and w.dtype == "bf16" and w.K <= 16:
+        return "softmax_smallk_kernel (8-CTA clusters, one pass over X)"
+    if w.loss == "softmax":
+        return "CUDA-core softmax gradient kernels"
+    return "grad_rows kernel with fused commit+decode (whole step)" if single else "grad_rows kernel"
 
 
 def load_peaks():
@@ -189,23 +211,52 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 
 def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 2):
-    """Steady steps/s of the oracle as it stands: warm-up step 0 untimed, then
-    steady steps until the budget is spent."""
+    """Steady steps/s of the oracle as it stands, and what was timed.
+
+    When the oracle's warm-up and two steady steps fit the budget, whole
+    steady steps are timed (warm-up step 0 untimed).  Otherwise a bounded
+    sample: the oracle's steady step is n partition gradients (each worker
+    evaluates its own) plus the literal decode (a c-slot coded sum per
+    received worker); partition gradients are timed one by one for about the
+    budget, one coded sum once, and the step time is n t_grad + (n - s) t_coded.
+    Returns (steps/s, count, seconds, sample description)."""
     from oracle import pgc_oracle as O
     S = {"FR": O.FR, "CR": O.CR}
     L = {"logistic": O.LOGISTIC, "lsq": O.LSQ, "softmax": O.SOFTMAX}
     Xf = [W.features_as_float(X, w.dtype) for X in Xs]
     o = O.PGCOracle(S[w.scheme], w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
-    o.step(masks[0])
+    t0 = time.perf_counter()
+    o.partition_grad(0)
+    t_pg = time.perf_counter() - t0
+    if t_pg * w.n * (w.c + 2) <= budget_s:
+        o.step(masks[0])
+        t0 = time.perf_counter()
+        k = 0
+        while True:
+            o.step(masks[(1 + k) % len(masks)])
+            k += 1
+            el = time.perf_counter() - t0
+            if (el >= budget_s and k >= min_steps) or el >= 4 * budget_s:
+                break
+        return k / el, k, el, f"{k} steady steps of the full {w.name} workload after the warm-up step ({el:.1f} s)"
+    # bounded sample
     t0 = time.perf_counter()
     k = 0
     while True:
-        o.step(masks[(1 + k) % len(masks)])
+        o.partition_grad(k % w.n)
         k += 1
         el = time.perf_counter() - t0
-        if (el >= budget_s and k >= min_steps) or el >= 4 * budget_s:
+        if (el >= budget_s and k >= 2) or k >= w.n:
             break
-    return k / el, k, el
+    t_grad = el / k
+    slots = [o.partition_grad(j % w.n) if j < 1 else np.ones_like(o.beta) for j in range(w.c)]
+    t1 = time.perf_counter()
+    _ = sum(slots[l] for l in range(w.c))
+    t_coded = time.perf_counter() - t1
+    step_s = w.n * t_grad + (w.n - w.s) * t_coded
+    desc = (f"{k} of the {w.n} partition gradients of one steady {w.name} step timed one by one ({el:.1f} s) "
+            f"plus one {w.c}-slot coded sum, scaled to n t_grad + (n - s) t_coded = {step_s:.2f} s per step")
+    return 1.0 / step_s, k, el, desc
 
 
 # ---------------------------------------------------------------------------
@@ -317,12 +368,18 @@ def run_ours(args):
     ms_per_step = max_over_ranks(ms_per_step, world, dev)
     value = world * 1000.0 / ms_per_step
 
-    # ---- roofline of the dominant kernel (the gradient kernel; when it
-    # carries the whole step, its launch duration is the step time) ---------
+    # ---- roofline of the dominant kernel (streaming paths: the gradient
+    # kernel, whose launch is the whole step when it carries the fused tail;
+    # tensor-core softmax: the slower of the two GEMMs) ----------------------
     peaks, peak_src = load_peaks()
     bound, units, unit, peak = roofline_model(w, peaks)
-    single = tim["launches"][1] == 0 and tim["launches"][2] == 0 and tim["launches"][0] == tim["steps"]
-    grad_ms = ms_per_step if (single and not flush) else tim["ms"][0] / max(1, tim["steps"])
+    nsteps = max(1, tim["steps"])
+    group_ms = [m / nsteps for m in tim["ms"]]
+    single = all(n == 0 for n in tim["launches"][1:]) and tim["launches"][0] == tim["steps"]
+    dom = 0
+    if tensor_core_path(w) and group_ms[2] > group_ms[0]:
+        dom = 2
+    grad_ms = ms_per_step if (single and not flush) else group_ms[dom]
     if unit == "GB/s":
         achieved = units / (grad_ms * 1e-3) / 1e9
     else:
@@ -345,10 +402,9 @@ def run_ours(args):
     # ---- cpu baseline (rank 0, N = 1 only) -------------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, k, el = time_oracle(w, Xs, ys, masks, args.cpu_seconds)
+        v, k, el, desc = time_oracle(w, Xs, ys, masks, args.cpu_seconds)
         cpu = {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
-               "sample": f"{k} steady steps of the full {w.name} workload after the warm-up step "
-                         f"({el:.1f} s, fp64 numpy, BLAS threads = all cores)"}
+               "sample": desc + "; fp64 numpy, BLAS threads = all cores"}
     g.close()
 
     uniq = evaluated_rows(w)
@@ -364,12 +420,12 @@ def run_ours(args):
                           f"inputs larger than L2: {step_bytes / 2**20:.0f} MiB streamed per step")},
         "samples_per_s_unique": value * uniq,
         "samples_per_s_worker": value * sum(w.rows()),
-        "kernel_ms_per_step": {KERNEL_NAMES[i]: tim["ms"][i] / max(1, tim["steps"]) for i in range(3)},
+        "kernel_ms_per_step": {B.KERNEL_GROUPS[i]: group_ms[i] for i in range(len(B.KERNEL_GROUPS))
+                               if tim["launches"][i] > 0},
         "kernel_timing_note": "per-group CUDA events from a separate pass; events between launches "
                               "serialise the dependent-launch overlap, so these sum to more than ms_per_step",
         "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
-                     "peak_source": peak_src, "kernel": ("gradient kernel with fused commit+decode (whole step)" if single else
-                                "gradient kernel") if w.loss != "softmax" else "gradient (softmax)",
+                     "peak_source": peak_src, "kernel": kernel_label(w, single, dom),
                      "duration_ms": grad_ms, "traffic": traffic,
                      "algorithmic_per_launch": units},
         "cpu_baseline": cpu,
@@ -394,7 +450,9 @@ def run_reference(args):
     Xs, ys = W.make_partitions(w, args.seed)
     masks = W.make_masks(w, K_steps + max(3, args.warmup) + 1, args.seed + 1000)
     budget = min(args.cpu_seconds, 60.0)
-    v, k, el = time_oracle(w, Xs, ys, masks, budget, min_steps=min(K_steps, 3))
+    v, k, el, desc = time_oracle(w, Xs, ys, masks, budget, min_steps=min(K_steps, 3))
+    if "steady steps" not in desc:
+        k = max(1, int(round(el * v)))         # sampled: whole-step equivalents of the timed work
     line = {
         "impl": "reference", "metric": METRIC, "value": v, "unit": "steps/s", "n_gpus": world, "steps": k,
         "warmup": 1, "ms_per_step": 1000.0 / v, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
@@ -402,7 +460,7 @@ def run_reference(args):
         "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
                    "rows_per_partition": w.m},
         "cpu_baseline": {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": f"{k} steady steps after the warm-up step ({el:.1f} s)"},
+                         "sample": desc},
         "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)

@@ -187,11 +187,16 @@ int64_t pgc_step_count(const pgc_ctx *ctx);
 
 /* ---- measurement ---------------------------------------------------------- */
 
-/* Kernel groups of one step, as counted and timed below. */
-#define PGC_KGRAD   0   /* per-partition gradient kernels                      */
-#define PGC_KCOMMIT 1   /* gradient-store commit                               */
-#define PGC_KDECODE 2   /* decode coefficients + decode + SGD                  */
-#define PGC_NKGROUPS 3
+/* Kernel groups of one step, in launch order, as counted and timed below.
+ * Paths without a group leave it empty (zero time, zero launches). */
+#define PGC_KGRAD   0   /* gradient: streaming row kernel, few-class softmax
+                           kernel, tensor-core logits GEMM, or the CUDA-core
+                           softmax kernels                                     */
+#define PGC_KRESID  1   /* tensor-core softmax: residual R = softmax(Z) - Y    */
+#define PGC_KGRADB  2   /* tensor-core softmax: gradient GEMM R^T X            */
+#define PGC_KCOMMIT 3   /* gradient-store commit                               */
+#define PGC_KDECODE 4   /* decode coefficients + decode + SGD                  */
+#define PGC_NKGROUPS 5
 
 /*
  * pgc_timing — enable != 0 starts recording CUDA events on the context's

@@ -70,6 +70,10 @@ for _name, (_res, _args) in _sig.items():
 EXPORTED = tuple(_sig)
 
 
+# kernel groups of one step, in launch order (PGC_KGRAD .. PGC_KDECODE)
+KERNEL_GROUPS = ("gradient", "residual", "gradient_backward", "commit", "decode")
+
+
 class PGCError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = code
@@ -245,9 +249,9 @@ class PGC:
         _check(lib.pgc_timing(self._h, 1 if enable else 0), "pgc_timing")
 
     def timing_read(self):
-        """Per kernel group (gradient, commit, decode): summed ms and launches."""
-        ms = (C.c_double * 3)()
-        nl = (_i64 * 3)()
+        """Per kernel group (KERNEL_GROUPS order): summed ms and launches."""
+        ms = (C.c_double * len(KERNEL_GROUPS))()
+        nl = (_i64 * len(KERNEL_GROUPS))()
         steps = _i64()
         _check(lib.pgc_timing_read(self._h, ms, nl, C.byref(steps)), "pgc_timing_read")
         return {"ms": list(ms), "launches": list(nl), "steps": steps.value}

@@ -637,7 +637,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
   cudaStream_t st = ctx->stream;
 
   PGC_CK(ctx, record_event(ctx));
-  int64_t nl[PGC_NKGROUPS] = {0, 0, 0};
+  int64_t nl[PGC_NKGROUPS] = {0, 0, 0, 0, 0};
   DecodeArgs dc;
   dc.scheme = ctx->scheme; dc.n = n; dc.s = ctx->s; dc.c = c; dc.slot = ph.slot; dc.owners = ctx->owners;
   dc.mask = bits; dc.P = ctx->P; dc.store = ctx->store; dc.U = ctx->U; dc.w = ctx->w; dc.wb = ctx->wb;
@@ -677,9 +677,11 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     f.a_off = ph.d_f_aoff; f.b_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back(); f.backward = 0;
     f.out_row0 = ph.d_f_outrow0; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
     PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, ctx->tmZo, nullptr, f, false, false, ctx->sm_count, st));
+    PGC_CK(ctx, record_event(ctx));
     PGC_CK(ctx, launch_softmax_bf16(ctx->Z, ctx->Rb, ctx->Ktc, ctx->K, static_cast<const int32_t*>(ctx->y),
                                     ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows,
                                     u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr, ctx->P, st));
+    PGC_CK(ctx, record_event(ctx));
     TcGemmParams b = {};
     b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.mt_count = ph.d_b_mvalid; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
     b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff; b.total_tiles = ph.b_prefix.back(); b.backward = 1;
@@ -688,7 +690,9 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     b.status = ctx->status; b.pdl = ctx->pdl ? 1 : 0;
     PGC_CK(ctx, launch_tc_gemm(ctx->tmR, ctx->tmXm, ctx->tmSo, ctx->tmUo, b, true, true, ctx->sm_count, st));
     dc.u_ready = u_red ? 1 : 0;
-    nl[PGC_KGRAD] = 3;
+    nl[PGC_KGRAD] = 1;
+    nl[PGC_KRESID] = 1;
+    nl[PGC_KGRADB] = 1;
     need_commit = false;
   } else if (ctx->smallk) {
     SmallKArgs a;
@@ -706,6 +710,10 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     a.Kpad = ctx->Kpad; a.partials = ctx->partials;
     nl[PGC_KGRAD] = 3;
     PGC_CK(ctx, launch_softmax_cc(a, st));
+  }
+  if (!ctx->tc) {
+    PGC_CK(ctx, record_event(ctx));   // empty residual and backward groups
+    PGC_CK(ctx, record_event(ctx));
   }
   PGC_CK(ctx, record_event(ctx));
   if (need_commit) {
@@ -822,9 +830,9 @@ int pgc_timing(pgc_ctx* ctx, int32_t enable) {
 int pgc_timing_read(pgc_ctx* ctx, double* ms, int64_t* launches, int64_t* steps_out) {
   if (!ctx) return PGC_EINVAL;
   PGC_CK(ctx, cudaStreamSynchronize(ctx->stream));
-  double acc[PGC_NKGROUPS] = {0, 0, 0};
-  // four events per recorded step: before grad, after grad, after commit, after decode
-  for (size_t i = 0; i + 3 < ctx->ev_used; i += 4) {
+  double acc[PGC_NKGROUPS] = {0, 0, 0, 0, 0};
+  // PGC_NKGROUPS + 1 events per recorded step: before the first group and after each
+  for (size_t i = 0; i + PGC_NKGROUPS < ctx->ev_used; i += PGC_NKGROUPS + 1) {
     for (int k = 0; k < PGC_NKGROUPS; ++k) {
       float t = 0.f;
       PGC_CK(ctx, cudaEventElapsedTime(&t, ctx->ev_pool[i + k], ctx->ev_pool[i + k + 1]));
