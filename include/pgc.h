@@ -168,6 +168,14 @@ int pgc_schedule(int32_t scheme, int32_t n, int32_t s, int64_t t,
 int pgc_get_store(pgc_ctx *ctx, int32_t worker, int32_t slot, float *out);
 
 /*
+ * pgc_get_store_cols — as pgc_get_store, for the parameters [col0, col0 +
+ * ncols) of the flattened K*d vector only (host out[ncols]); reads a few
+ * columns of every store without copying whole gradients.  Errors:
+ * PGC_EINVAL (range outside [0, K*d)), PGC_ESTATE, PGC_ECUDA.
+ */
+int pgc_get_store_cols(pgc_ctx *ctx, int32_t worker, int32_t slot, int64_t col0, int64_t ncols, float *out);
+
+/*
  * pgc_get_decode — the decoding coefficients the device derived from the
  * last step's mask: coeff[i] (host [n]) = weight a_i of W_i's coded gradient
  * (§IV-A: 1/n for each FR group's representative; §V-B: 1/((n-s)c) for each

@@ -54,6 +54,7 @@ _sig = {
     "pgc_placement": (C.c_int, [_i32, _i32, _i32, C.POINTER(_i32)]),
     "pgc_schedule": (C.c_int, [_i32, _i32, _i32, _i64, C.POINTER(_i32), C.POINTER(_i32)]),
     "pgc_get_store": (C.c_int, [_vp, _i32, _i32, C.POINTER(C.c_float)]),
+    "pgc_get_store_cols": (C.c_int, [_vp, _i32, _i32, _i64, _i64, C.POINTER(C.c_float)]),
     "pgc_get_decode": (C.c_int, [_vp, C.POINTER(C.c_float)]),
     "pgc_get_weights": (C.c_int, [_vp, C.POINTER(C.c_float)]),
     "pgc_set_weights": (C.c_int, [_vp, C.POINTER(C.c_float)]),
@@ -234,6 +235,13 @@ class PGC:
     def decode_coefficients(self) -> np.ndarray:
         out = np.zeros(self.n, dtype=np.float32)
         _check(lib.pgc_get_decode(self._h, out.ctypes.data_as(C.POINTER(C.c_float))), "pgc_get_decode")
+        return out
+
+    def store_cols(self, worker: int, slot: int, col0: int, ncols: int) -> np.ndarray:
+        """Columns [col0, col0 + ncols) of the flattened K*d stored gradient."""
+        out = np.empty(ncols, dtype=np.float32)
+        _check(lib.pgc_get_store_cols(self._h, worker, slot, col0, ncols, out.ctypes.data_as(C.POINTER(C.c_float))),
+               "pgc_get_store_cols")
         return out
 
     def weights(self) -> np.ndarray:

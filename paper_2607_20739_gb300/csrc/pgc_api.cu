@@ -789,6 +789,24 @@ int pgc_get_store(pgc_ctx* ctx, int32_t worker, int32_t slot, float* out) {
   return read_status(ctx);
 }
 
+int pgc_get_store_cols(pgc_ctx* ctx, int32_t worker, int32_t slot, int64_t col0, int64_t ncols, float* out) {
+  if (!ctx || !out || worker < 0 || worker >= ctx->n || slot < 0 || slot >= ctx->c) return PGC_EINVAL;
+  if (col0 < 0 || ncols < 0 || col0 + ncols > ctx->K * ctx->d) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  const int owner = ctx->scheme == PGC_FR ? worker / ctx->c : worker;
+  const float* src = ctx->store + ((size_t)owner * ctx->c + slot) * ctx->P;
+  // flattened index k*d + j lives at k*ld + j: one copy per class row touched
+  int64_t done = 0;
+  while (done < ncols) {
+    const int64_t col = col0 + done, k = col / ctx->d, j = col % ctx->d;
+    const int64_t len = std::min<int64_t>(ncols - done, ctx->d - j);
+    PGC_CK(ctx, cudaMemcpyAsync(out + done, src + k * ctx->ld + j, (size_t)len * sizeof(float),
+                                cudaMemcpyDeviceToHost, ctx->stream));
+    done += len;
+  }
+  return read_status(ctx);
+}
+
 int pgc_get_decode(pgc_ctx* ctx, float* coeff) {
   if (!ctx || !coeff) return PGC_EINVAL;
   if (!ctx->stepped || ctx->broken) return PGC_ESTATE;
