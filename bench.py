@@ -407,6 +407,18 @@ def run_ours(args):
                "sample": desc + "; fp64 numpy, BLAS threads = all cores"}
     g.close()
 
+    # ---- simulated wall clock of a step (the paper's time per step, PGC vs
+    # DGD / IS-SGD / GC): measured compute and decode, seeded delays in units
+    # of the compute time --------------------------------------------------
+    from paper_2607_20739_gb300 import wallclock as WC
+    compute_s = sum(group_ms[:3]) * 1e-3
+    decode_s = sum(group_ms[3:]) * 1e-3
+    delays = W.draw_delays(w, K_steps + Wu + 1, args.seed + 1000)[Wu:Wu + K_steps]
+    sim = WC.summary(delays, w.n, w.s, compute_s, compute_s, decode_s)
+    sim["model"] = ("each worker finishes after (partitions evaluated) x compute + delay; the master waits for "
+                    "the n - s fastest (pgc, is_sgd, gc with c partitions per worker) or all n (dgd), then decodes; "
+                    "delays are the seeded draws that pick the stragglers, in units of the compute time")
+
     uniq = evaluated_rows(w)
     line = {
         "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K_steps, "warmup": Wu,
@@ -432,6 +444,7 @@ def run_ours(args):
         "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": w.n,
                 "d2h_bytes_per_step": 2 * P * 4},
         "gpu_launches": int(round(launches_per_step * K_steps)),
+        "simulated_wall_clock": sim,
         "clocks": clocks,
     }
     if rank == 0:
