@@ -49,6 +49,8 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=W.WORKLOAD_ORDER)
     ap.add_argument("--seed", type=int, default=1)
+    ap.add_argument("--mode", default="pgc", choices=["pgc", "is_sgd", "gc"],
+                    help="training scheme on the same kernels: PGC, or the IS-SGD / GC (FR) baselines")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle sample")
     ap.add_argument("--override", action="append", default=[],
@@ -210,7 +212,7 @@ class ClockSampler:
 # the fp64 oracle on the host cores (cpu_baseline and --impl reference)
 # ---------------------------------------------------------------------------
 
-def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 2):
+def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 2, mode: str = "pgc"):
     """Steady steps/s of the oracle as it stands, and what was timed.
 
     When the oracle's warm-up and two steady steps fit the budget, whole
@@ -224,11 +226,16 @@ def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 
     S = {"FR": O.FR, "CR": O.CR}
     L = {"logistic": O.LOGISTIC, "lsq": O.LSQ, "softmax": O.SOFTMAX}
     Xf = [W.features_as_float(X, w.dtype) for X in Xs]
-    o = O.PGCOracle(S[w.scheme], w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
+    if mode == "pgc":
+        o = O.PGCOracle(S[w.scheme], w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
+    else:
+        o = {"is_sgd": O.ISSGDOracle, "gc": O.GCFROracle}[mode](w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
+    inner = o if mode == "pgc" else o.inner
+    evals_per_step = w.n * (w.c if mode == "gc" else 1)
     t0 = time.perf_counter()
-    o.partition_grad(0)
+    inner.partition_grad(0)
     t_pg = time.perf_counter() - t0
-    if t_pg * w.n * (w.c + 2) <= budget_s:
+    if t_pg * (w.n * w.c + 2 * evals_per_step) <= budget_s:
         o.step(masks[0])
         t0 = time.perf_counter()
         k = 0
@@ -243,19 +250,20 @@ def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 
     t0 = time.perf_counter()
     k = 0
     while True:
-        o.partition_grad(k % w.n)
+        inner.partition_grad(k % w.n)
         k += 1
         el = time.perf_counter() - t0
-        if (el >= budget_s and k >= 2) or k >= w.n:
+        if (el >= budget_s and k >= 2) or k >= evals_per_step:
             break
     t_grad = el / k
-    slots = [o.partition_grad(j % w.n) if j < 1 else np.ones_like(o.beta) for j in range(w.c)]
+    nslot = 1 if mode == "is_sgd" else w.c                 # gradients per uploaded (coded) gradient
+    slots = [inner.partition_grad(j % w.n) if j < 1 else np.ones_like(inner.beta) for j in range(nslot)]
     t1 = time.perf_counter()
-    _ = sum(slots[l] for l in range(w.c))
+    _ = sum(slots[l] for l in range(nslot))
     t_coded = time.perf_counter() - t1
-    step_s = w.n * t_grad + (w.n - w.s) * t_coded
-    desc = (f"{k} of the {w.n} partition gradients of one steady {w.name} step timed one by one ({el:.1f} s) "
-            f"plus one {w.c}-slot coded sum, scaled to n t_grad + (n - s) t_coded = {step_s:.2f} s per step")
+    step_s = evals_per_step * t_grad + (w.n - w.s) * t_coded
+    desc = (f"{k} of the {evals_per_step} partition gradients of one steady {w.name} step timed one by one ({el:.1f} s) "
+            f"plus one {nslot}-slot coded sum, scaled to (evaluations) t_grad + (n - s) t_coded = {step_s:.2f} s per step")
     return 1.0 / step_s, k, el, desc
 
 
@@ -313,7 +321,7 @@ def run_ours(args):
     masks = W.make_masks(w, K_steps + Wu + 1, args.seed + 1000)
 
     stream = torch.cuda.Stream(device=dev)
-    g = B.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream)
+    g = B.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream, mode=args.mode)
     g.load(Xs, ys)
     P = w.K * w.d
     gout = torch.empty(P, device=dev)
@@ -402,7 +410,7 @@ def run_ours(args):
     # ---- cpu baseline (rank 0, N = 1 only) -------------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, k, el, desc = time_oracle(w, Xs, ys, masks, args.cpu_seconds)
+        v, k, el, desc = time_oracle(w, Xs, ys, masks, args.cpu_seconds, mode=args.mode)
         cpu = {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": desc + "; fp64 numpy, BLAS threads = all cores"}
     g.close()
@@ -411,7 +419,8 @@ def run_ours(args):
     # DGD / IS-SGD / GC): measured compute and decode, seeded delays in units
     # of the compute time --------------------------------------------------
     from paper_2607_20739_gb300 import wallclock as WC
-    compute_s = sum(group_ms[:3]) * 1e-3
+    # one partition per worker: a GC run measures c partitions per worker
+    compute_s = sum(group_ms[:3]) * 1e-3 / (w.c if args.mode == "gc" else 1)
     decode_s = sum(group_ms[3:]) * 1e-3
     delays = W.draw_delays(w, K_steps + Wu + 1, args.seed + 1000)[Wu:Wu + K_steps]
     sim = WC.summary(delays, w.n, w.s, compute_s, compute_s, decode_s)
@@ -427,7 +436,7 @@ def run_ours(args):
         "data": f"synthetic, seeded (seed {args.seed}); {w.features} features, planted-model labels, "
                 f"{w.delays} straggler delays",
         "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
-                   "rows_per_partition": w.m, "features": w.dtype, "parallelism": f"replicas{world}",
+                   "rows_per_partition": w.m, "features": w.dtype, "parallelism": f"replicas{world}", "mode": args.mode,
                    "l2": ("flushed between steps (256 MiB write, excluded from step time)" if flush else
                           f"inputs larger than L2: {step_bytes / 2**20:.0f} MiB streamed per step")},
         "samples_per_s_unique": value * uniq,
@@ -463,7 +472,7 @@ def run_reference(args):
     Xs, ys = W.make_partitions(w, args.seed)
     masks = W.make_masks(w, K_steps + max(3, args.warmup) + 1, args.seed + 1000)
     budget = min(args.cpu_seconds, 60.0)
-    v, k, el, desc = time_oracle(w, Xs, ys, masks, budget, min_steps=min(K_steps, 3))
+    v, k, el, desc = time_oracle(w, Xs, ys, masks, budget, min_steps=min(K_steps, 3), mode=args.mode)
     if "steady steps" not in desc:
         k = max(1, int(round(el * v)))         # sampled: whole-step equivalents of the timed work
     line = {
@@ -471,7 +480,7 @@ def run_reference(args):
         "warmup": 1, "ms_per_step": 1000.0 / v, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f64", "data": f"synthetic, seeded (seed {args.seed})",
         "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
-                   "rows_per_partition": w.m},
+                   "rows_per_partition": w.m, "mode": args.mode},
         "cpu_baseline": {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -82,6 +82,28 @@ int pgc_create(pgc_ctx **out, int32_t n, int32_t s, int32_t scheme, int32_t loss
                int32_t dtype, int64_t d, int64_t K, const int64_t *rows, float lr,
                const float *w0, void *stream);
 
+/* Training schemes on the same kernels (§VI-A, the paper's baselines). */
+#define PGC_MODE_PGC    0   /* pipelined gradient coding (default)                  */
+#define PGC_MODE_IS_SGD 1   /* ignore stragglers: worker W_i evaluates D_i each step;
+                               the master averages the n - s received gradients.
+                               Needs scheme PGC_CR (the decode runs as CR with one
+                               slot per worker, coefficient 1/(n - s)).             */
+#define PGC_MODE_GC     2   /* gradient coding with fractional repetition: every
+                               worker evaluates all c partitions of its group each
+                               step; the master decodes one coded gradient per group
+                               (1/n), which recovers (1/n) sum_k g_k exactly.  Needs
+                               scheme PGC_FR (GC-CR's coefficients are only cited). */
+
+/*
+ * pgc_create_mode — pgc_create with a training scheme from PGC_MODE_*; the
+ * other arguments and errors are pgc_create's (PGC_EINVAL also for an unknown
+ * mode or a mode/scheme pair listed as unsupported above).  With s = 0 every
+ * mode is plain distributed gradient descent (DGD, §III).
+ */
+int pgc_create_mode(pgc_ctx **out, int32_t mode, int32_t n, int32_t s, int32_t scheme, int32_t loss,
+                    int32_t dtype, int64_t d, int64_t K, const int64_t *rows, float lr,
+                    const float *w0, void *stream);
+
 /*
  * pgc_load_partitions — copy the n partitions into device memory (§III: the
  * partitions are placed before training).  X[k] points to [m_k][d] features

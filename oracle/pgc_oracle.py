@@ -35,6 +35,10 @@ Readings where the paper is silent (each is also listed in the design notes):
   R7  losses: logistic cross-entropy with y in {0, 1}; least squares
       (1/2)(x.beta - y)^2; softmax cross-entropy; no bias, no regulariser.
 
+Baselines (§VI-A), for comparison on the same kernels: IS-SGD (the master
+averages the n - s fastest workers' own-partition gradients) and GC with FR
+placement (every worker evaluates its c partitions every step).
+
 Parity of whole trajectories is pinned only through the invariants the paper
 proves (eq. cr-fullsum, eq. cr-unbiased, the FR / GC equivalence and the DGD
 special case); there is no printed trajectory to compare with.
@@ -333,6 +337,101 @@ class PGCOracle:
         rec["beta"] = self.beta.copy()
         self.t = t + 1
         return rec
+
+
+# ----------------------------------------------------------------------------
+# The paper's baselines on the same problem (§VI-A), literally per worker
+# ----------------------------------------------------------------------------
+
+class ISSGDOracle:
+    """Ignore-stragglers SGD (§VI-A): every step worker W_i evaluates the
+    gradient of its own partition D_i at beta^(t); the master averages the
+    gradients of the n - s fastest workers and ignores the rest."""
+
+    def __init__(self, n, s, loss, Xs, ys, lr, beta0=None, K=1):
+        self.inner = PGCOracle(CR, n, 0, loss, Xs, ys, lr, beta0=beta0, K=K)   # data, beta, gradients
+        self.n, self.s = n, s
+        self.t = 0
+
+    @property
+    def beta(self):
+        return self.inner.beta
+
+    def step(self, mask):
+        check_mask(mask, self.n, self.s)
+        R = received_set(mask)
+        a = np.zeros(self.n)
+        for i in R:
+            a[i] = 1.0 / len(R)                 # mean of the n - s received gradients
+        g = np.zeros_like(self.inner.beta)
+        for i in range(self.n):
+            gi = self.inner.partition_grad(i)   # stragglers compute too; their result is not used
+            if a[i] != 0.0:
+                g = g + a[i] * gi
+        rec = {"t": self.t, "slot": 0, "eval_partition": list(range(self.n)), "fr_rep": None, "coeff": a,
+               "received": len(R), "grad": g}
+        self.inner.beta = self.inner.beta - self.inner.lr * g
+        rec["beta"] = self.inner.beta.copy()
+        self.t += 1
+        return rec
+
+    def loss_value(self):
+        return self.inner.loss_value()
+
+
+class GCFROracle:
+    """Gradient coding with fractional repetition (§VI-A, the GC baseline; the
+    FR construction of §IV-A with every gradient current): every step each
+    worker evaluates all c partitions of its group at beta^(t) and uploads
+    their sum; the master takes one coded gradient per group, from its
+    lowest-index non-straggler, and scales the sum by 1/n."""
+
+    def __init__(self, n, s, loss, Xs, ys, lr, beta0=None, K=1):
+        self.inner = PGCOracle(FR, n, 0, loss, Xs, ys, lr, beta0=beta0, K=K)
+        self.n, self.s, self.c = n, s, s + 1
+        if n % self.c:
+            raise ValueError("FR needs c | n")
+        self.hold = holdings(FR, n, self.c)
+        self.t = 0
+
+    @property
+    def beta(self):
+        return self.inner.beta
+
+    def step(self, mask):
+        check_mask(mask, self.n, self.s)
+        coded = [sum(self.inner.partition_grad(k) for k in self.hold[i]) for i in range(self.n)]
+        reps = fr_representatives(mask, self.n, self.c)
+        a = np.zeros(self.n)
+        for r in reps:
+            a[r] = 1.0 / self.n
+        g = np.zeros_like(self.inner.beta)
+        for r in reps:
+            g = g + a[r] * coded[r]
+        rec = {"t": self.t, "slot": -1, "eval_partition": [-1] * self.n, "fr_rep": reps, "coeff": a,
+               "received": self.n - self.s, "grad": g}
+        self.inner.beta = self.inner.beta - self.inner.lr * g
+        rec["beta"] = self.inner.beta.copy()
+        self.t += 1
+        return rec
+
+    def loss_value(self):
+        return self.inner.loss_value()
+
+
+def run_mode(mode, scheme, n, s, loss, Xs, ys, lr, masks, beta0=None, K=1, record_loss=True):
+    """run() for a training mode: "pgc", "is_sgd" or "gc" (GC with FR placement)."""
+    if mode == "pgc":
+        return run(scheme, n, s, loss, Xs, ys, lr, masks, beta0=beta0, K=K, record_loss=record_loss)
+    cls = {"is_sgd": ISSGDOracle, "gc": GCFROracle}[mode]
+    o = cls(n, s, loss, Xs, ys, lr, beta0=beta0, K=K)
+    out = []
+    for mask in masks:
+        lv = o.loss_value() if record_loss else None
+        rec = o.step(mask)
+        rec["loss"] = lv
+        out.append(rec)
+    return out
 
 
 def run(scheme, n, s, loss, Xs, ys, lr, masks, beta0=None, K=1, record_loss=True):

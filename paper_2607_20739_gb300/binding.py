@@ -32,6 +32,8 @@ F32, BF16 = 0, 1
 SCHEMES = {"FR": FR, "CR": CR}
 LOSSES = {"logistic": LOGISTIC, "lsq": LSQ, "softmax": SOFTMAX}
 DTYPES = {"f32": F32, "bf16": BF16}
+MODE_PGC, MODE_IS_SGD, MODE_GC = 0, 1, 2
+MODES = {"pgc": MODE_PGC, "is_sgd": MODE_IS_SGD, "gc": MODE_GC}
 
 
 class StepInfo(C.Structure):
@@ -44,6 +46,8 @@ _i32 = C.c_int32
 _i64 = C.c_int64
 _sig = {
     "pgc_create": (C.c_int, [C.POINTER(_vp), _i32, _i32, _i32, _i32, _i32, _i64, _i64, C.POINTER(_i64), C.c_float,
+                             C.POINTER(C.c_float), _vp]),
+    "pgc_create_mode": (C.c_int, [C.POINTER(_vp), _i32, _i32, _i32, _i32, _i32, _i32, _i64, _i64, C.POINTER(_i64), C.c_float,
                              C.POINTER(C.c_float), _vp]),
     "pgc_load_partitions": (C.c_int, [_vp, C.POINTER(_vp), C.POINTER(_vp), _i32]),
     "pgc_step": (C.c_int, [_vp, C.POINTER(C.c_uint8), _vp, _vp, _i32, C.POINTER(StepInfo)]),
@@ -131,11 +135,13 @@ class PGC:
     """One PGC run on the current CUDA device (a ``pgc_ctx``)."""
 
     def __init__(self, scheme, n: int, s: int, loss, dtype, d: int, K: int = 1, rows=None, lr: float = 0.1,
-                 w0=None, stream=None):
+                 w0=None, stream=None, mode="pgc"):
         self.scheme = _enum(scheme, SCHEMES)
         self.loss_kind = _enum(loss, LOSSES)
         self.dtype = _enum(dtype, DTYPES)
-        self.n, self.s, self.c, self.d, self.K = n, s, s + 1, d, K
+        self.mode = _enum(mode, MODES)
+        c = 1 if self.mode == MODE_IS_SGD else s + 1
+        self.n, self.s, self.c, self.d, self.K = n, s, c, d, K
         rows = np.asarray(rows if rows is not None else [1] * n, dtype=np.int64)
         if rows.shape != (n,):
             raise ValueError("rows must have one entry per partition")
@@ -146,9 +152,9 @@ class PGC:
             w0p = w0.ctypes.data_as(C.POINTER(C.c_float))
         self._stream = _stream_handle(stream)
         h = _vp()
-        _check(lib.pgc_create(C.byref(h), n, s, self.scheme, self.loss_kind, self.dtype, d, K,
-                              rows.ctypes.data_as(C.POINTER(_i64)), C.c_float(lr), w0p, _vp(self._stream)),
-               "pgc_create")
+        _check(lib.pgc_create_mode(C.byref(h), self.mode, n, s, self.scheme, self.loss_kind, self.dtype, d, K,
+                                   rows.ctypes.data_as(C.POINTER(_i64)), C.c_float(lr), w0p, _vp(self._stream)),
+               "pgc_create_mode")
         self._h = h
         self._mask = np.zeros(n, dtype=np.uint8)
         self._eval = np.zeros(n, dtype=np.int32)

@@ -116,6 +116,7 @@ struct pgc_ctx {
                              // work-item counter, finished producers (zero between steps)
   bool pdl = true;           // chain the step's kernels with programmatic dependent launch
   int tail_mode = 0;         // fused tail of the gradient kernel (see GradRowsArgs)
+  int mode = PGC_MODE_PGC;   // training scheme (PGC_MODE_*)
   bool tc = false;           // softmax on the tensor cores (bf16 features)
   bool smallk = false;       // few-class softmax: one-pass cluster kernel
   int sk_nper = 0;           // its 64-feature blocks per CTA slice
@@ -371,10 +372,19 @@ int pgc_schedule(int32_t scheme, int32_t n, int32_t s, int64_t t, int32_t* eval_
 
 int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss, int32_t dtype, int64_t d,
                int64_t K, const int64_t* rows, float lr, const float* w0, void* stream) {
+  return pgc_create_mode(out, PGC_MODE_PGC, n, s, scheme, loss, dtype, d, K, rows, lr, w0, stream);
+}
+
+int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t scheme, int32_t loss,
+                    int32_t dtype, int64_t d, int64_t K, const int64_t* rows, float lr, const float* w0,
+                    void* stream) {
   if (!out) return PGC_EINVAL;
   *out = nullptr;
   int rc = check_nsc(scheme, n, s);
   if (rc) return rc;
+  if (mode != PGC_MODE_PGC && mode != PGC_MODE_IS_SGD && mode != PGC_MODE_GC) return PGC_EINVAL;
+  if (mode == PGC_MODE_IS_SGD && scheme != PGC_CR) return PGC_EINVAL;
+  if (mode == PGC_MODE_GC && scheme != PGC_FR) return PGC_EINVAL;
   if (!valid_loss(loss) || !valid_dtype(dtype) || d < 1 || !rows || !std::isfinite(lr)) return PGC_EINVAL;
   if (loss == PGC_SOFTMAX ? (K < 2 || K > 4096) : K != 1) return PGC_EINVAL;
   for (int k = 0; k < n; ++k)
@@ -383,7 +393,10 @@ int pgc_create(pgc_ctx** out, int32_t n, int32_t s, int32_t scheme, int32_t loss
 
   pgc_ctx* ctx = new (std::nothrow) pgc_ctx();
   if (!ctx) return PGC_ENOMEM;
-  ctx->n = n; ctx->s = s; ctx->c = s + 1; ctx->scheme = scheme; ctx->loss = loss; ctx->dtype = dtype;
+  // IS-SGD keeps one slot per worker (its own partition) and still ignores s stragglers
+  ctx->mode = mode;
+  ctx->n = n; ctx->s = s; ctx->c = mode == PGC_MODE_IS_SGD ? 1 : s + 1;
+  ctx->scheme = scheme; ctx->loss = loss; ctx->dtype = dtype;
   ctx->d = d; ctx->K = K; ctx->lr = lr;
   ctx->stream = static_cast<cudaStream_t>(stream);
   ctx->esize = dtype == PGC_BF16 ? 2 : 4;
@@ -632,7 +645,11 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
   if (cnt != ctx->s) return PGC_EMASK;
 
   const int64_t t = ctx->t;
-  const int pidx = t == 0 ? 0 : 1 + (int)((t - 1) % c);
+  // GC refreshes every slot every step (the warm-up phase); IS-SGD's one slot
+  // is refreshed every step, t = 0 included
+  const int pidx = ctx->mode == PGC_MODE_GC ? 0
+                   : ctx->mode == PGC_MODE_IS_SGD ? 1
+                   : t == 0 ? 0 : 1 + (int)((t - 1) % c);
   Phase& ph = ctx->phases[pidx];
   cudaStream_t st = ctx->stream;
 

@@ -40,19 +40,20 @@ def oracle_inputs(w: W.Workload, Xs):
     return [W.features_as_float(X, w.dtype) for X in Xs]
 
 
-def run_oracle(w: W.Workload, Xs, ys, masks, record_loss=True):
-    return O.run(SCHEME[w.scheme], w.n, w.s, LOSS[w.loss], oracle_inputs(w, Xs), ys, w.lr, list(masks),
-                 K=w.K, record_loss=record_loss)
+def run_oracle(w: W.Workload, Xs, ys, masks, record_loss=True, mode="pgc"):
+    return O.run_mode(mode, SCHEME[w.scheme], w.n, w.s, LOSS[w.loss], oracle_inputs(w, Xs), ys, w.lr, list(masks),
+                      K=w.K, record_loss=record_loss)
 
 
-def make_gpu(binding, w: W.Workload, Xs, ys, stream=None):
-    g = binding.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream)
+def make_gpu(binding, w: W.Workload, Xs, ys, stream=None, mode="pgc"):
+    g = binding.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream,
+                    mode=mode)
     g.load(Xs, ys)
     return g
 
 
-def run_gpu(binding, w: W.Workload, Xs, ys, masks, record_loss=True):
-    g = make_gpu(binding, w, Xs, ys)
+def run_gpu(binding, w: W.Workload, Xs, ys, masks, record_loss=True, mode="pgc"):
+    g = make_gpu(binding, w, Xs, ys, mode=mode)
     P = w.K * w.d
     out = []
     for mask in masks:
