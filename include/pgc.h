@@ -212,6 +212,28 @@ int pgc_get_weights(pgc_ctx *ctx, float *out);
  * tests; also the checkpoint-restore path).  Errors: PGC_EINVAL, PGC_ECUDA. */
 int pgc_set_weights(pgc_ctx *ctx, const float *w);
 
+/*
+ * Checkpoint and resume of a run: the step counter t, beta, every store
+ * (owners x c gradients) and the slot totals U — everything a later step
+ * reads.  The features and labels are not part of it: the resumed context
+ * must be created with the same arguments and loaded with the same
+ * partitions.
+ *
+ * pgc_checkpoint_bytes — *bytes = size of the checkpoint of this context:
+ *   104 bytes of header (13 int64: magic 0x3154504B43434750 "PGCCKPT1",
+ *   version 1, mode, scheme, loss, dtype, n, s, c, d, K, t, stepped) then fp32
+ *   beta [K][d], stores [owners][c][K][d] and U [c][K][d], host byte order.
+ * pgc_checkpoint_save — write it to host buf[bytes] (waits for the stream).
+ * pgc_checkpoint_load — restore it from host buf[bytes] into a context with
+ *   the same mode, scheme, loss, dtype, n, s, d and K; the next pgc_step is
+ *   step t of the saved run.
+ * Errors: PGC_EINVAL (NULL, wrong size, header of another configuration),
+ * PGC_ESTATE (a failed context), PGC_ECUDA.
+ */
+int pgc_checkpoint_bytes(pgc_ctx *ctx, int64_t *bytes);
+int pgc_checkpoint_save(pgc_ctx *ctx, void *buf, int64_t bytes);
+int pgc_checkpoint_load(pgc_ctx *ctx, const void *buf, int64_t bytes);
+
 /* pgc_step_count — number of steps taken so far (host-side counter). */
 int64_t pgc_step_count(const pgc_ctx *ctx);
 

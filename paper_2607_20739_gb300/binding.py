@@ -58,6 +58,9 @@ _sig = {
     "pgc_placement": (C.c_int, [_i32, _i32, _i32, C.POINTER(_i32)]),
     "pgc_schedule": (C.c_int, [_i32, _i32, _i32, _i64, C.POINTER(_i32), C.POINTER(_i32)]),
     "pgc_get_store": (C.c_int, [_vp, _i32, _i32, C.POINTER(C.c_float)]),
+    "pgc_checkpoint_bytes": (C.c_int, [_vp, C.POINTER(_i64)]),
+    "pgc_checkpoint_save": (C.c_int, [_vp, _vp, _i64]),
+    "pgc_checkpoint_load": (C.c_int, [_vp, _vp, _i64]),
     "pgc_get_store_cols": (C.c_int, [_vp, _i32, _i32, _i64, _i64, C.POINTER(C.c_float)]),
     "pgc_get_decode": (C.c_int, [_vp, C.POINTER(C.c_float)]),
     "pgc_get_weights": (C.c_int, [_vp, C.POINTER(C.c_float)]),
@@ -249,6 +252,19 @@ class PGC:
         _check(lib.pgc_get_store_cols(self._h, worker, slot, col0, ncols, out.ctypes.data_as(C.POINTER(C.c_float))),
                "pgc_get_store_cols")
         return out
+
+    def checkpoint(self) -> np.ndarray:
+        """The run's state (t, beta, stores, slot totals) as a host byte array."""
+        nb = _i64()
+        _check(lib.pgc_checkpoint_bytes(self._h, C.byref(nb)), "pgc_checkpoint_bytes")
+        buf = np.empty(nb.value, dtype=np.uint8)
+        _check(lib.pgc_checkpoint_save(self._h, buf.ctypes.data, nb.value), "pgc_checkpoint_save")
+        return buf
+
+    def restore(self, buf) -> None:
+        """Resume from checkpoint(): the next step is the saved run's next step."""
+        b = np.ascontiguousarray(np.asarray(buf, dtype=np.uint8))
+        _check(lib.pgc_checkpoint_load(self._h, b.ctypes.data, b.size), "pgc_checkpoint_load")
 
     def weights(self) -> np.ndarray:
         out = np.zeros(self.K * self.d, dtype=np.float32)

@@ -848,6 +848,72 @@ int pgc_set_weights(pgc_ctx* ctx, const float* w) {
   return read_status(ctx);
 }
 
+// ---- checkpoint --------------------------------------------------------------
+namespace {
+constexpr int64_t kCkptMagic = 0x3154504B43434750LL;   // "PGCCKPT1" little-endian
+constexpr int kCkptHeader = 13;
+int64_t ckpt_bytes(const pgc_ctx* ctx) {
+  const int64_t Kd = ctx->K * ctx->d;
+  return kCkptHeader * 8 + 4 * (Kd + (int64_t)ctx->owners * ctx->c * Kd + (int64_t)ctx->c * Kd);
+}
+void ckpt_header(const pgc_ctx* ctx, int64_t* h) {
+  const int64_t v[kCkptHeader] = {kCkptMagic, 1, ctx->mode, ctx->scheme, ctx->loss, ctx->dtype, ctx->n, ctx->s,
+                                  ctx->c, ctx->d, ctx->K, ctx->t, ctx->stepped ? 1 : 0};
+  for (int i = 0; i < kCkptHeader; ++i) h[i] = v[i];
+}
+}  // namespace
+
+int pgc_checkpoint_bytes(pgc_ctx* ctx, int64_t* bytes) {
+  if (!ctx || !bytes) return PGC_EINVAL;
+  *bytes = ckpt_bytes(ctx);
+  return PGC_OK;
+}
+
+int pgc_checkpoint_save(pgc_ctx* ctx, void* buf, int64_t bytes) {
+  if (!ctx || !buf || bytes != ckpt_bytes(ctx)) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  int64_t* h = static_cast<int64_t*>(buf);
+  ckpt_header(ctx, h);
+  float* p = reinterpret_cast<float*>(h + kCkptHeader);
+  const int64_t Kd = ctx->K * ctx->d;
+  int rc = copy_out(ctx, p, ctx->w, 0);
+  if (rc) return rc;
+  p += Kd;
+  for (int64_t r = 0; r < (int64_t)ctx->owners * ctx->c; ++r, p += Kd)
+    if ((rc = copy_out(ctx, p, ctx->store + r * ctx->P, 0))) return rc;
+  for (int o = 0; o < ctx->c; ++o, p += Kd)
+    if ((rc = copy_out(ctx, p, ctx->U + (int64_t)o * ctx->P, 0))) return rc;
+  return read_status(ctx);
+}
+
+int pgc_checkpoint_load(pgc_ctx* ctx, const void* buf, int64_t bytes) {
+  if (!ctx || !buf || bytes != ckpt_bytes(ctx)) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  const int64_t* h = static_cast<const int64_t*>(buf);
+  int64_t want[kCkptHeader];
+  ckpt_header(ctx, want);
+  // magic, version and the configuration must match; t and stepped are restored
+  for (int i = 0; i < kCkptHeader - 2; ++i)
+    if (h[i] != want[i]) return PGC_EINVAL;
+  if (h[11] < 0) return PGC_EINVAL;
+  const float* p = reinterpret_cast<const float*>(h + kCkptHeader);
+  const int64_t Kd = ctx->K * ctx->d;
+  auto copy_in = [&](float* dst, const float* src) {
+    return cudaMemcpy2DAsync(dst, ctx->ld * sizeof(float), src, ctx->d * sizeof(float), ctx->d * sizeof(float),
+                             ctx->K, cudaMemcpyHostToDevice, ctx->stream);
+  };
+  PGC_CK(ctx, copy_in(ctx->w, p));
+  p += Kd;
+  for (int64_t r = 0; r < (int64_t)ctx->owners * ctx->c; ++r, p += Kd) PGC_CK(ctx, copy_in(ctx->store + r * ctx->P, p));
+  for (int o = 0; o < ctx->c; ++o, p += Kd) PGC_CK(ctx, copy_in(ctx->U + (int64_t)o * ctx->P, p));
+  if (ctx->wb) PGC_CK(ctx, launch_f32_to_bf16(ctx->w, ctx->wb, ctx->P, ctx->stream));
+  const int rc = read_status(ctx);
+  if (rc) return rc;
+  ctx->t = h[11];
+  ctx->stepped = h[12] != 0;
+  return PGC_OK;
+}
+
 int64_t pgc_step_count(const pgc_ctx* ctx) { return ctx ? ctx->t : -1; }
 
 int pgc_timing(pgc_ctx* ctx, int32_t enable) {
