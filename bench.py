@@ -288,6 +288,12 @@ def max_over_ranks(value: float, world: int, device=None) -> float:
     return float(t.item())
 
 
+def job_value(ms_per_step_max: float, world: int) -> float:
+    """Whole-job steps/s: every replica runs its own copy of the workload
+    (weak scaling), so the job completes `world` steps per slowest-rank step."""
+    return world * 1000.0 / ms_per_step_max
+
+
 def barrier(world: int):
     if world > 1:
         import torch.distributed as dist
@@ -374,7 +380,7 @@ def run_ours(args):
     else:
         ms_per_step = region_ms / K_steps
     ms_per_step = max_over_ranks(ms_per_step, world, dev)
-    value = world * 1000.0 / ms_per_step
+    value = job_value(ms_per_step, world)
 
     # ---- roofline of the dominant kernel (streaming paths: the gradient
     # kernel, whose launch is the whole step when it carries the fused tail;
