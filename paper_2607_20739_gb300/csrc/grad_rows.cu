@@ -49,7 +49,6 @@ constexpr int kNT = kNW * 32;          // consumer threads
 constexpr int kThreads = kNT + 64;     // + a producer warp + a tail warp
 constexpr int kProducer = kNT;        // producer thread
 constexpr int kTailWarp = kNW + 1;     // warp index of the tail warp
-constexpr int64_t kPrefetchBytes = 256 * 1024;   // L2 warm-up per CTA at start
 constexpr int64_t kPrefetchChunkRows = 16;
 
 struct StageHdr {
@@ -189,13 +188,14 @@ __device__ void produce(const GradRowsArgs& a, const Smem& sm, const StageCfg& c
   bool ok = true, waited = false;
   int item = blockIdx.x;
   if (item < a.nitems) {
-    // Beyond the S stages it can hold, warm L2 with the next rows of the
-    // first item: a CTA started early by the dependent launch keeps HBM busy
-    // while the previous step finishes, and reads these rows from L2 later.
+    // Beyond the S stages it can hold, optionally warm L2 with the next rows
+    // of the first item while the previous step finishes (a.prefetch_bytes;
+    // on the streaming workloads this traffic slowed the previous step's
+    // serial tail more than it saved, so the library passes 0).
     const WorkItem it = a.items[item];
     const int64_t r0 = it.row0 + (int64_t)c.S * c.SR;
     int64_t rows = it.rows - (int64_t)c.S * c.SR;
-    const int64_t cap = (int64_t)(kPrefetchBytes / rb);
+    const int64_t cap = a.prefetch_bytes / rb;
     rows = rows < cap ? rows : cap;
     for (int64_t r = 0; r < rows; r += kPrefetchChunkRows) {
       const int64_t n = rows - r < kPrefetchChunkRows ? rows - r : kPrefetchChunkRows;

@@ -117,6 +117,7 @@ struct pgc_ctx {
   bool pdl = true;           // chain the step's kernels with programmatic dependent launch
   int tail_mode = 0;         // fused tail of the gradient kernel (see GradRowsArgs)
   int mode = PGC_MODE_PGC;   // training scheme (PGC_MODE_*)
+  int64_t prefetch_bytes = 0;  // streaming kernel's L2 warm-up per CTA (PGC_PREFETCH_KB)
   bool tc = false;           // softmax on the tensor cores (bf16 features)
   bool smallk = false;       // few-class softmax: one-pass cluster kernel
   int sk_nper = 0;           // its 64-feature blocks per CTA slice
@@ -425,6 +426,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   }
   ctx->P = ctx->K * ctx->ld;
   ctx->Kpad = (int64_t)align_up((size_t)K, 4);
+  if (const char* env = std::getenv("PGC_PREFETCH_KB")) ctx->prefetch_bytes = (int64_t)std::atoll(env) * 1024;
   {
     const char* env = std::getenv("PGC_NO_PDL");
     ctx->pdl = !(env && env[0] == '1');
@@ -673,6 +675,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     g.items = ph.d_items; g.nitems = (int)ph.items.size(); g.max_item_rows = ph.max_item_rows;
     g.partials = ctx->partials; g.status = ctx->status;
     g.tail = ph.tail; g.pdl = ctx->pdl;
+    g.prefetch_bytes = ctx->prefetch_bytes;
     g.cnt_e = ctx->counters; g.cnt_all = ctx->counters + n;
     g.work_ctr = ctx->counters + n + 1; g.prod_done = ctx->counters + n + 2; g.grid = ctx->sm_count;
     g.e_item0 = ph.d_e_item0; g.e_scale = ph.d_e_scale; g.e_dest = ph.d_e_dest; g.ndest = ph.ndest;

@@ -89,6 +89,7 @@ struct GradRowsArgs {
   int nE = 0;
   float* store = nullptr;   // [owners * c][ld]
   DecodeArgs dec;           // used when tail == 2
+  int64_t prefetch_bytes = 0; // L2 warm-up per CTA before waiting for the previous step
 };
 int grad_rows_variant(int dtype, int64_t d, int64_t* ld_out);  // chooses ld, returns variant id
 int grad_rows_stage_rows(int variant, int64_t ld, int dtype);
