@@ -112,8 +112,12 @@ def roofline_model(w: W.Workload, peaks: dict):
 
 def kernel_label(w: W.Workload, single: bool, dom: int) -> str:
     if tensor_core_path(w):
-        return ("tc_gemm_kernel, gradient R^T X" if dom == 2 else "tc_gemm_kernel, logits X W^T") + \
-            " (tcgen05, 2-CTA clusters)"
+        nt = -(-w.K // 256)
+        if dom == 2:
+            return "tc_gemm_kernel, gradient R^T X (tcgen05, 2-CTA clusters)"
+        if nt in (1, 2, 4, 8):
+            return f"tc_logits_softmax_kernel, logits X W^T + softmax residual (tcgen05, {nt}-CTA clusters)"
+        return "tc_gemm_kernel, logits X W^T (tcgen05, 2-CTA clusters)"
     if w.loss == "softmax" and w.dtype == "bf16" and w.K <= 16:
         return "softmax_smallk_kernel (8-CTA clusters, one pass over X)"
     if w.loss == "softmax":

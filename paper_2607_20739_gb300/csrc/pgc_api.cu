@@ -51,6 +51,9 @@ struct Phase {
   int32_t *d_f_prefix = nullptr, *d_f_nk = nullptr, *d_f_aoff = nullptr, *d_f_mvalid = nullptr;
   int32_t *d_b_prefix = nullptr, *d_b_nk = nullptr, *d_b_aoff = nullptr, *d_b_boff = nullptr, *d_b_mvalid = nullptr;
   int64_t* d_f_outrow0 = nullptr;
+  // fused logits + residual kernel: 128-row tiles {X row, R row, valid rows, e}
+  std::vector<int32_t> q_tiles;
+  int32_t* d_q_tiles = nullptr;
   // few-class softmax: 128-row tiles {row0, rows, item, flags} and items
   std::vector<int32_t> sk_tiles;
   int sk_items = 0;
@@ -132,6 +135,10 @@ struct pgc_ctx {
   alignas(64) unsigned char tmZo[128];   // Z fp32 output     (box 32 x 32)
   alignas(64) unsigned char tmSo[128];   // stores [slot][K][ld] fp32 output (box 32 x 32 x 1)
   alignas(64) unsigned char tmUo[128];   // U [c][K][ld] fp32, reduce-add target
+  bool tcf = false;          // logits GEMM with the residual fused (no Z in HBM)
+  int tcf_nc = 0;            // its clusters of Ktc / 256 CTAs
+  alignas(64) unsigned char tmXq[128];   // X as the fused kernel's A part (box 64 x 128/NT)
+  alignas(64) unsigned char tmRst[128];  // Rb as the fused kernel's output (box 64 x 32)
   int64_t loss_chunk = 0;
   int loss_nblocks = 256;
   void* tables = nullptr;
@@ -275,6 +282,12 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
       for (int e = 0; e < nE; ++e) {
         const int64_t m = ph.e_rows[e];
         ph.e_zrow0p.push_back(zp);
+        for (int64_t r = 0; r < m; r += 128) {
+          ph.q_tiles.push_back((int32_t)(ph.e_row0[e] + r));
+          ph.q_tiles.push_back((int32_t)(zp + r));
+          ph.q_tiles.push_back((int32_t)std::min<int64_t>(128, m - r));
+          ph.q_tiles.push_back(e);
+        }
         ph.f_nk.push_back((int32_t)(ctx->ld / 64));
         ph.f_aoff.push_back((int32_t)ph.e_row0[e]);
         ph.f_outrow0.push_back(zp);
@@ -417,6 +430,13 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     ctx->tc = dtype == PGC_BF16 && K >= kTcMinClasses && K <= kTcMaxClasses && !(env && env[0] == '1');
     ctx->ld = (int64_t)align_up((size_t)d, ctx->tc ? 256 : 64);
     ctx->Ktc = (int64_t)align_up((size_t)K, 256);
+    // the residual runs in the logits GEMM's epilogue when one cluster can
+    // hold every class of a row tile (PGC_NO_FUSED=1 keeps three kernels)
+    const char* env3 = std::getenv("PGC_NO_FUSED");
+    if (ctx->tc && !(env3 && env3[0] == '1')) {
+      ctx->tcf_nc = tc_softmax_max_clusters((int)(ctx->Ktc / 256));
+      ctx->tcf = ctx->tcf_nc > 0;
+    }
     const char* env2 = std::getenv("PGC_NO_SMALLK");
     if (!ctx->tc && dtype == PGC_BF16 && !(env2 && env2[0] == '1') && smallk_fits(K, ctx->ld)) {
       ctx->sk_nper = (int)((ctx->ld / 64 + 7) / 8);
@@ -462,7 +482,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   std::vector<uint8_t> tab;
   size_t off = 0;
   std::vector<size_t> offs;
-  constexpr int kTabs = 19;
+  constexpr int kTabs = 20;
   for (auto& ph : ctx->phases) {
     offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
@@ -483,6 +503,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_boff);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_mvalid);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.sk_tiles);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.q_tiles);
   }
   // loss chunks (softmax): {row0, rows, 0} per chunk
   std::vector<int64_t> ldesc;
@@ -523,7 +544,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   for (auto& ph : ctx->phases) max_zpad = std::max(max_zpad, ph.zpad_total);
   if (loss == PGC_SOFTMAX) {
     const size_t zcc = (size_t)std::max<int64_t>(max_z, ctx->loss_chunk) * ctx->Kpad;
-    const size_t ztc = ctx->tc ? (size_t)max_zpad * ctx->Ktc : 0;
+    const size_t ztc = ctx->tc && !ctx->tcf ? (size_t)max_zpad * ctx->Ktc : 0;
     PGC_ALLOC(ctx->Z, std::max(zcc, ztc) * sizeof(float));
   }
   if (ctx->tc) PGC_ALLOC(ctx->Rb, (size_t)max_zpad * ctx->Ktc * sizeof(uint16_t));
@@ -576,6 +597,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     ph.d_b_boff = reinterpret_cast<int32_t*>(base + o[16]);
     ph.d_b_mvalid = reinterpret_cast<int32_t*>(base + o[17]);
     ph.d_sk_tiles = reinterpret_cast<int32_t*>(base + o[18]);
+    ph.d_q_tiles = reinterpret_cast<int32_t*>(base + o[19]);
   }
   ctx->loss_desc = nullptr;
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
@@ -595,8 +617,12 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     const uint64_t sd[3] = {(uint64_t)ctx->ld, (uint64_t)ctx->K, (uint64_t)ctx->owners * ctx->c};
     const uint64_t ud[3] = {(uint64_t)ctx->ld, (uint64_t)ctx->K, (uint64_t)ctx->c};
     const uint64_t ss[2] = {(uint64_t)ctx->ld * 4, (uint64_t)ctx->P * 4};
-    ok = ok && make_tmap_f32_box32(ctx->tmZo, ctx->Z, 2, zd, zs) && make_tmap_f32_box32(ctx->tmSo, ctx->store, 3, sd, ss) &&
-         make_tmap_f32_box32(ctx->tmUo, ctx->U, 3, ud, ss);
+    ok = ok && make_tmap_f32_box32(ctx->tmSo, ctx->store, 3, sd, ss) && make_tmap_f32_box32(ctx->tmUo, ctx->U, 3, ud, ss);
+    if (ctx->tcf)
+      ok = ok && make_tmap_bf16(ctx->tmXq, ctx->X, ctx->ld, ctx->total_rows, pitch, (uint32_t)(128 / (ctx->Ktc / 256))) &&
+           make_tmap_bf16(ctx->tmRst, ctx->Rb, ctx->Ktc, max_zpad, (uint64_t)ctx->Ktc * 2, 32);
+    else
+      ok = ok && make_tmap_f32_box32(ctx->tmZo, ctx->Z, 2, zd, zs);
     if (!ok) return fail(cudaErrorInvalidValue);
   }
 #undef PGC_ALLOC
@@ -696,12 +722,25 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     const bool u_red = ph.slot >= 0 && ph.ndest == 1;
     f.a_off = ph.d_f_aoff; f.b_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back(); f.backward = 0;
     f.out_row0 = ph.d_f_outrow0; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
-    PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, ctx->tmZo, nullptr, f, false, false, ctx->sm_count, st));
-    PGC_CK(ctx, record_event(ctx));
-    PGC_CK(ctx, launch_softmax_bf16(ctx->Z, ctx->Rb, ctx->Ktc, ctx->K, static_cast<const int32_t*>(ctx->y),
-                                    ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows,
-                                    u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr, ctx->P, st));
-    PGC_CK(ctx, record_event(ctx));
+    if (ctx->tcf) {
+      // R straight from the logits GEMM's epilogue
+      TcSoftmaxParams q = {};
+      q.tiles = reinterpret_cast<const int4*>(ph.d_q_tiles); q.ntiles = (int)(ph.q_tiles.size() / 4);
+      q.NT = (int)(ctx->Ktc / 256); q.nk = (int)(ctx->ld / 64); q.K = (int)ctx->K;
+      q.y = static_cast<const int32_t*>(ctx->y);
+      q.zero_buf = u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr; q.zero_n4 = ctx->P / 4;
+      q.status = ctx->status; q.pdl = ctx->pdl ? 1 : 0;
+      PGC_CK(ctx, launch_tc_softmax(ctx->tmXq, ctx->tmW, ctx->tmRst, q, ctx->tcf_nc, st));
+      PGC_CK(ctx, record_event(ctx));
+      PGC_CK(ctx, record_event(ctx));   // empty residual group
+    } else {
+      PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, ctx->tmZo, nullptr, f, false, false, ctx->sm_count, st));
+      PGC_CK(ctx, record_event(ctx));
+      PGC_CK(ctx, launch_softmax_bf16(ctx->Z, ctx->Rb, ctx->Ktc, ctx->K, static_cast<const int32_t*>(ctx->y),
+                                      ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows,
+                                      u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr, ctx->P, st));
+      PGC_CK(ctx, record_event(ctx));
+    }
     TcGemmParams b = {};
     b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.mt_count = ph.d_b_mvalid; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
     b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff; b.total_tiles = ph.b_prefix.back(); b.backward = 1;
@@ -711,7 +750,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     PGC_CK(ctx, launch_tc_gemm(ctx->tmR, ctx->tmXm, ctx->tmSo, ctx->tmUo, b, true, true, ctx->sm_count, st));
     dc.u_ready = u_red ? 1 : 0;
     nl[PGC_KGRAD] = 1;
-    nl[PGC_KRESID] = 1;
+    nl[PGC_KRESID] = ctx->tcf ? 0 : 1;
     nl[PGC_KGRADB] = 1;
     need_commit = false;
   } else if (ctx->smallk) {

@@ -199,6 +199,29 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
                                 const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
                                 int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st);
 
+// ---- tensor-core logits GEMM with the softmax residual in its epilogue ------
+// (tc_softmax.cu) for every 128-row tile {first X row, first R row, valid
+// rows, partition}: R[r][k] = softmax_k(X Wb^T)[r] - [k == y_r] as bf16, rows
+// past `valid` zero.  A cluster of NT = Ktc / 256 CTAs (1, 2, 4 or 8) covers
+// all classes of one tile; also zeroes zero_buf[0 : 4 zero_n4].
+struct TcSoftmaxParams {
+  const int4* tiles;
+  int ntiles;
+  int NT;                   // CTAs per cluster (256 classes each)
+  int nk;                   // ld / 64
+  int K;
+  const int32_t* y;         // labels per global X row
+  float* zero_buf;
+  int64_t zero_n4;
+  int* status;
+  int pdl;
+};
+// Clusters of NT that fit at once (0: this NT is not supported).
+int tc_softmax_max_clusters(int NT);
+// tmXq: X, box {64, 128 / NT}; tmW: Wb, box {64, 128}; tmR: Rb, box {64, 32}
+cudaError_t launch_tc_softmax(const void* tmXq, const void* tmW, const void* tmR, const TcSoftmaxParams& p,
+                              int nclusters, cudaStream_t st);
+
 // ---- softmax with few classes: one pass over X per step --------------------
 // tiles[i] = {first global X row, rows (<= kSmallKRows), item, flags: 1 first / 2 last
 // tile of a cluster's run in one partition}; cluster c of nc takes tiles

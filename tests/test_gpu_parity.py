@@ -40,6 +40,10 @@ CASES = {
     "fr_tc_k256_unequal_rows": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=256, d=600,
                                                                      m=(130, 1, 64, 257)), 5),
     "cr_tc_k128_c_equals_n": (WL["cr_n128_softmax_k1000"].replace(n=3, s=2, K=128, d=256, m=300), 5),
+    # fused logits + residual with 8-CTA clusters (K > 1792), and K = 1500
+    # (six 256-class tiles: the three-kernel path)
+    "cr_tc_k2000_nt8": (WL["cr_n128_softmax_k1000"].replace(n=3, s=1, K=2000, d=300, m=150), 4),
+    "fr_tc_k1500_unfused": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=1500, d=256, m=(90, 200, 3, 128)), 4),
     # few-class softmax (one-pass cluster kernel): ragged tiles, partition
     # boundaries inside a cluster's run, empty feature slices, K = 16
     "fr_smallk_k10_unequal_rows": (WL["fr_n32_softmax_k10"].replace(n=4, s=1, d=3072, m=(300, 1, 129, 700)), 5),
