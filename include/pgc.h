@@ -161,6 +161,11 @@ int pgc_destroy(pgc_ctx *ctx);
 /* pgc_strerror — static text for a status code. */
 const char *pgc_strerror(int32_t code);
 
+/* pgc_last_cuda_error — name of the CUDA runtime error behind the most
+ * recent PGC_ECUDA / PGC_ENOMEM returned on the calling thread (for example
+ * "cudaErrorLaunchOutOfResources"), or "" if there was none.  Static text. */
+const char *pgc_last_cuda_error(void);
+
 /* ---- host-only helpers: pure index arithmetic, no CUDA call ------------- */
 
 /*

@@ -55,6 +55,7 @@ _sig = {
     "pgc_sync": (C.c_int, [_vp]),
     "pgc_destroy": (C.c_int, [_vp]),
     "pgc_strerror": (C.c_char_p, [_i32]),
+    "pgc_last_cuda_error": (C.c_char_p, []),
     "pgc_placement": (C.c_int, [_i32, _i32, _i32, C.POINTER(_i32)]),
     "pgc_schedule": (C.c_int, [_i32, _i32, _i32, _i64, C.POINTER(_i32), C.POINTER(_i32)]),
     "pgc_get_store": (C.c_int, [_vp, _i32, _i32, C.POINTER(C.c_float)]),
@@ -85,7 +86,12 @@ KERNEL_GROUPS = ("gradient", "residual", "gradient_backward", "commit", "decode"
 class PGCError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = code
-        super().__init__(f"{where}: {lib.pgc_strerror(code).decode()} ({code})")
+        msg = f"{where}: {lib.pgc_strerror(code).decode()} ({code})"
+        if code in (ECUDA, ENOMEM):
+            name = lib.pgc_last_cuda_error().decode()
+            if name:
+                msg += f" [{name}]"
+        super().__init__(msg)
 
 
 def _check(code: int, where: str) -> None:

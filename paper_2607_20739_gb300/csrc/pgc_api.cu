@@ -54,6 +54,9 @@ struct Phase {
   // fused logits + residual kernel: 128-row tiles {X row, R row, valid rows, e}
   std::vector<int32_t> q_tiles;
   int32_t* d_q_tiles = nullptr;
+  // gradient contraction: units {class pair tile, feature tile, first e, run length}
+  std::vector<int32_t> g_units;
+  int32_t* d_g_units = nullptr;
   // few-class softmax: 128-row tiles {row0, rows, item, flags} and items
   std::vector<int32_t> sk_tiles;
   int sk_items = 0;
@@ -137,6 +140,7 @@ struct pgc_ctx {
   alignas(64) unsigned char tmUo[128];   // U [c][K][ld] fp32, reduce-add target
   bool tcf = false;          // logits GEMM with the residual fused (no Z in HBM)
   int tcf_nc = 0;            // its clusters of Ktc / 256 CTAs
+  int tcg_pairs = 0;         // co-resident CTA pairs of the gradient contraction
   alignas(64) unsigned char tmXq[128];   // X as the fused kernel's A part (box 64 x 128/NT)
   alignas(64) unsigned char tmRst[128];  // Rb as the fused kernel's output (box 64 x 32)
   int64_t loss_chunk = 0;
@@ -158,8 +162,11 @@ struct pgc_ctx {
 
 namespace {
 
+thread_local cudaError_t g_last_cuda_error = cudaSuccess;
+
 int cuda_fail(pgc_ctx* ctx, cudaError_t e) {
   if (e == cudaSuccess) return PGC_OK;
+  g_last_cuda_error = e;
   if (ctx) ctx->broken = true;
   return e == cudaErrorMemoryAllocation ? PGC_ENOMEM : PGC_ECUDA;
 }
@@ -302,6 +309,29 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
         zp += (m + 127) / 128 * 128;   // whole forward tiles: their TMA stores stay inside the partition
       }
       ph.zpad_total = zp;
+      // gradient units: every (class pair tile, feature tile) for runs of gs
+      // consecutive partitions; gs balances the rounds over the CTA pairs
+      // (ties go to the longer run: fewer reduce-adds into U) while a run's
+      // inputs stay well inside L2
+      const int64_t PT = (int64_t)(MTb / 2) * NTb, np = std::max(1, ctx->tcg_pairs);
+      const double per_part = (double)ph.max_rows * (double)(ctx->ld + ctx->Ktc) * 2.0;
+      int gs = 1;
+      int64_t best = INT64_MAX;
+      for (int g = 1; g <= kTcGradMaxRun; ++g) {
+        if (g > 1 && g * per_part > 48.0 * 1024 * 1024) break;
+        const int64_t units = (nE + g - 1) / g * PT;
+        const int64_t cost = (units + np - 1) / np * g;
+        if (cost <= best) { best = cost; gs = g; }
+      }
+      if (const char* env = std::getenv("PGC_GRAD_RUN")) gs = std::min(kTcGradMaxRun, std::max(1, std::atoi(env)));
+      for (int e0 = 0; e0 < nE; e0 += gs)
+        for (int mp = 0; mp < MTb / 2; ++mp)
+          for (int nt = 0; nt < NTb; ++nt) {
+            ph.g_units.push_back(mp);
+            ph.g_units.push_back(nt);
+            ph.g_units.push_back(e0);
+            ph.g_units.push_back(std::min(gs, nE - e0));
+          }
     }
   }
 }
@@ -346,6 +376,10 @@ int copy_out(pgc_ctx* ctx, float* dst, const float* src, int on_device) {
 }  // namespace
 
 extern "C" {
+
+const char* pgc_last_cuda_error(void) {
+  return g_last_cuda_error == cudaSuccess ? "" : cudaGetErrorName(g_last_cuda_error);
+}
 
 const char* pgc_strerror(int32_t code) {
   switch (code) {
@@ -433,6 +467,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     // the residual runs in the logits GEMM's epilogue when one cluster can
     // hold every class of a row tile (PGC_NO_FUSED=1 keeps three kernels)
     const char* env3 = std::getenv("PGC_NO_FUSED");
+    if (ctx->tc) ctx->tcg_pairs = tc_grad_max_pairs();
     if (ctx->tc && !(env3 && env3[0] == '1')) {
       ctx->tcf_nc = tc_softmax_max_clusters((int)(ctx->Ktc / 256));
       ctx->tcf = ctx->tcf_nc > 0;
@@ -482,7 +517,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   std::vector<uint8_t> tab;
   size_t off = 0;
   std::vector<size_t> offs;
-  constexpr int kTabs = 20;
+  constexpr int kTabs = 21;
   for (auto& ph : ctx->phases) {
     offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
@@ -504,6 +539,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_mvalid);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.sk_tiles);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.q_tiles);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.g_units);
   }
   // loss chunks (softmax): {row0, rows, 0} per chunk
   std::vector<int64_t> ldesc;
@@ -598,6 +634,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     ph.d_b_mvalid = reinterpret_cast<int32_t*>(base + o[17]);
     ph.d_sk_tiles = reinterpret_cast<int32_t*>(base + o[18]);
     ph.d_q_tiles = reinterpret_cast<int32_t*>(base + o[19]);
+    ph.d_g_units = reinterpret_cast<int32_t*>(base + o[20]);
   }
   ctx->loss_desc = nullptr;
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
@@ -741,13 +778,13 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
                                       u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr, ctx->P, st));
       PGC_CK(ctx, record_event(ctx));
     }
-    TcGemmParams b = {};
-    b.nbatch = nE; b.tile_prefix = ph.d_b_prefix; b.mt_count = ph.d_b_mvalid; b.NT = (int)(ctx->ld / 256); b.nk = ph.d_b_nk;
-    b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff; b.total_tiles = ph.b_prefix.back(); b.backward = 1;
+    TcGradParams b = {};
+    b.units = reinterpret_cast<const int4*>(ph.d_g_units); b.nunits = (int)(ph.g_units.size() / 4);
+    b.nk = ph.d_b_nk; b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff;
     b.scale = ph.d_e_scale; b.dest = ph.d_e_dest; b.ndest = ph.ndest; b.m_limit = (int)ctx->K;
     b.u_reduce = u_red ? 1 : 0; b.u_slot = ph.slot;
     b.status = ctx->status; b.pdl = ctx->pdl ? 1 : 0;
-    PGC_CK(ctx, launch_tc_gemm(ctx->tmR, ctx->tmXm, ctx->tmSo, ctx->tmUo, b, true, true, ctx->sm_count, st));
+    PGC_CK(ctx, launch_tc_grad(ctx->tmR, ctx->tmXm, ctx->tmSo, ctx->tmUo, b, ctx->tcg_pairs, st));
     dc.u_ready = u_red ? 1 : 0;
     nl[PGC_KGRAD] = 1;
     nl[PGC_KRESID] = ctx->tcf ? 0 : 1;

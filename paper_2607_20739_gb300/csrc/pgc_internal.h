@@ -199,6 +199,34 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
                                 const int64_t* e_row0, const int64_t* e_rows, const int64_t* e_zrow0, int nE,
                                 int64_t max_rows, float* zero_buf, int64_t zero_n, cudaStream_t st);
 
+// ---- tensor-core gradient contraction (tc_grad.cu) -------------------------
+// G_e = scale_e R_e^T X_e for the runs of partitions in `units`
+// ({class pair tile mp, feature tile nt, first batch, batches}), written as
+// 32 x 32 fp32 boxes into the stores [slot][K][ld] (3-D map) at every dest of
+// the batch; with u_reduce each run's sum is also added (TMA reduce-add) into
+// U [c][K][ld] at u_slot.  R is read as MN-major A (box 64 x 64), X as
+// MN-major B (box 64 x 64).
+struct TcGradParams {
+  const int4* units;
+  int nunits;
+  const int* nk;            // [nbatch] K blocks of 64 rows (ceil(m_e / 64))
+  const int* a_off;         // [nbatch] first R row of the batch
+  const int* b_off;         // [nbatch] first X row of the batch
+  const float* scale;       // [nbatch] 1/m_e
+  const int32_t* dest;      // [nbatch * ndest] store index or -1
+  int ndest;
+  int m_limit;              // classes that exist (K); boxes past it are skipped
+  int u_reduce;
+  int u_slot;
+  int* status;
+  int pdl;
+};
+constexpr int kTcGradMaxRun = 8;   // partitions per unit at most
+// Clusters of two that fit at once (0: the kernel cannot be launched).
+int tc_grad_max_pairs();
+cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmS, const void* tmU, const TcGradParams& p,
+                           int npairs, cudaStream_t st);
+
 // ---- tensor-core logits GEMM with the softmax residual in its epilogue ------
 // (tc_softmax.cu) for every 128-row tile {first X row, first R row, valid
 // rows, partition}: R[r][k] = softmax_k(X Wb^T)[r] - [k == y_r] as bf16, rows

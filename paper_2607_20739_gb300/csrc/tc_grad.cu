@@ -1,0 +1,342 @@
+// Gradient contraction of the tensor-core softmax path (§III with f = log
+// sum_k exp(w_k.x) - w_y.x): for every evaluated partition e,
+//
+//   G_e[k][j] = (1/m_e) sum_{r in D_e} R[r][k] X[r][j]     A = R (MN-major), B = X (MN-major)
+//
+// written straight into every store that keeps the partition, and, in steady
+// steps, the slot total U[o_t] = sum_e G_e (§V-B) formed on the way out.
+//
+// Work is split into units {pair tile, run of partitions}: a cluster of two
+// CTAs owns the 256 x 256 output tile (class tiles 2mp, 2mp+1; feature tile
+// nt) for a run of up to eight partitions and computes G_e of each in turn.
+// Each CTA loads its 128 x 64 R tile and one half of the 64 x 256 X tile,
+// multicast into both CTAs, into a 4-stage ring (2-D TMA, 128-byte swizzle);
+// warp 1 issues tcgen05.mma (M = 128 classes, N = 256 features, K = 16 rows)
+// into one of two TMEM accumulators.  Eight epilogue warps (two per TMEM lane
+// quarter, 128 columns each) drain the other: the scaled gradient goes out as
+// 32 x 32 fp32 boxes with TMA stores (evict-first: the stores are only read
+// back for stragglers), and each thread keeps its row's share of the run's
+// sum in registers, added into U[o_t] with one TMA reduce-add per box at the
+// end of the run.  So U costs one reduce per run instead of one per partition.
+// Every wait is bounded; the TMEM allocation is released on every path.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+
+#include "tc_common.cuh"
+
+namespace pgc {
+
+namespace {
+
+constexpr int kGM = 128, kGN = 256, kGK = 64;
+constexpr int kGS = 4;                          // shared-memory stages
+constexpr uint32_t kGA = kGM * kGK * 2;         // 16 KB R tile (two 64 x 64 boxes)
+constexpr uint32_t kGB = kGN * kGK * 2;         // 32 KB X tile (four 64 x 64 boxes)
+constexpr int kGThreads = 320;                  // producer, MMA, 8 epilogue warps
+constexpr int kGEpi = 8;
+constexpr uint32_t kGTmem = 2 * kGN;            // two fp32 accumulators
+constexpr uint32_t kGBox = 32 * 32 * 4;         // one 32 x 32 fp32 output box
+
+struct GradSmem {
+  uint32_t sA, sB, box, bars, total;
+};
+__host__ __device__ constexpr GradSmem grad_smem() {
+  return GradSmem{0, kGS * kGA, kGS * (kGA + kGB), kGS * (kGA + kGB) + kGEpi * kGBox,
+                  kGS * (kGA + kGB) + kGEpi * kGBox + 16 * 8};
+}
+
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+
+// stage 16 values (columns 16 half .. 16 half + 15) of this lane's row into
+// its 128-byte row of a swizzled box (16-byte chunk c at c ^ (row & 7))
+__device__ __forceinline__ void stage_half(uint8_t* box, int lane, int half, const float* v) {
+  float4* rowp = reinterpret_cast<float4*>(box + lane * 128);
+#pragma unroll
+  for (int c = 0; c < 4; ++c)
+    rowp[(4 * half + c) ^ (lane & 7)] = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+}
+
+}  // namespace
+
+// Ten warps put three on some of the SM's four register-file quarters, so a
+// thread gets at most 168 registers; the epilogue keeps 128 partial sums of
+// the slot total in them and reads TMEM 16 columns at a time.
+__global__ void __launch_bounds__(kGThreads, 1)
+tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmX,
+               const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmU, TcGradParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr GradSmem L = grad_smem();
+  uint8_t* sA = sm + L.sA;
+  uint8_t* sB = sm + L.sB;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.bars);
+  uint64_t* full = bars;                // [4]
+  uint64_t* empty = bars + 4;           // [4]
+  uint64_t* acc_full = bars + 8;        // [2]
+  uint64_t* acc_empty = bars + 10;      // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  int* cta_err = reinterpret_cast<int*>(bars + 13);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rank = (int)cluster_rank();
+  constexpr uint16_t kPair = 0x3;
+  if (threadIdx.x == 0) {
+    *cta_err = 0;
+    for (int s = 0; s < kGS; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 2);           // the MMAs of both CTAs read the stage
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], kGEpi);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kGTmem)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  cluster_sync_all();                    // the peer's barriers exist before any multicast
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  if (threadIdx.x == 0) grid_dep_launch();
+  if (p.pdl) grid_dep_wait();           // R is the previous kernel's output; U was zeroed there
+
+  const int pair = (int)blockIdx.x >> 1, npairs = (int)gridDim.x >> 1;
+  const int my_units = p.nunits > pair ? (p.nunits - pair + npairs - 1) / npairs : 0;
+
+  if (warp == 0 && lane == 0) {
+    // ---- producer ----------------------------------------------------------
+    int it = 0;
+    bool ok = true;
+    for (int i = 0; i < my_units && ok; ++i) {
+      const int4 u = p.units[pair + i * npairs];
+      const int mt = 2 * u.x + rank, nt = u.y;
+      for (int j = 0; j < u.w && ok; ++j) {
+        const int b = u.z + j;
+        const int nkb = p.nk[b];
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % kGS;
+          if (it >= kGS && !mbar_wait(&empty[s], ((it / kGS) - 1) & 1, p.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[s], kGA + kGB);
+          uint8_t* a_dst = sA + (size_t)s * kGA;
+          uint8_t* b_dst = sB + (size_t)s * kGB;
+          for (int q = 0; q < 2; ++q)
+            tma_load_2d(a_dst + q * 8192, &tmR, mt * kGM + q * 64, p.a_off[b] + kb * kGK, &full[s]);
+          for (int q = 2 * rank; q < 2 * rank + 2; ++q)
+            tma_load_2d_mc(b_dst + q * 8192, &tmX, nt * kGN + q * 64, p.b_off[b] + kb * kGK, &full[s], kPair);
+        }
+      }
+    }
+    if (!ok) atomicExch(cta_err, 1);
+    // no copy may outlive the CTA: wait for the last fill of every stage
+    for (int s = 0; s < kGS && s < it; ++s) {
+      const int last = ((it - 1 - s) / kGS) * kGS + s;
+      mbar_wait(&full[s], (last / kGS) & 1, p.status);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---- MMA issuer --------------------------------------------------------
+    constexpr uint32_t idesc = idesc_bf16_f32(kGM, kGN, true, true);
+    int it = 0, tt = 0;
+    bool ok = true;
+    for (int i = 0; i < my_units && ok; ++i) {
+      const int4 u = p.units[pair + i * npairs];
+      for (int j = 0; j < u.w && ok; ++j, ++tt) {
+        const int acc = tt & 1;
+        if (tt >= 2 && !mbar_wait(&acc_empty[acc], ((tt / 2) - 1) & 1, p.status)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + (uint32_t)(acc * kGN);
+        const int nkb = p.nk[u.z + j];
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const int s = it % kGS;
+          if (!mbar_wait(&full[s], (it / kGS) & 1, p.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(sA + (size_t)s * kGA);
+          const uint32_t b_base = smem_u32(sB + (size_t)s * kGB);
+#pragma unroll
+          for (int kk = 0; kk < kGK / 16; ++kk) {
+            // MN-major: the next 16 K rows are two 8-row groups (2 KB) further
+            const uint64_t da = smem_desc_sw128(a_base + kk * 2048, 8192, 1024);
+            const uint64_t db = smem_desc_sw128(b_base + kk * 2048, 8192, 1024);
+            umma_bf16(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit_mc(&empty[s], kPair);  // this CTA is done with the stage, in both CTAs' count
+        }
+        if (!ok) break;
+        umma_commit(&acc_full[acc]);     // the accumulator is complete
+      }
+    }
+    if (!ok) atomicExch(cta_err, 1);
+  } else if (warp >= 2) {
+    // ---- epilogue ----------------------------------------------------------
+    // Warp w drains TMEM lanes 32q..32q+31 (q = w % 4: the lane quarter it may
+    // read), columns 128h..128h+127, 32 at a time, into its 32 x 32 box of
+    // shared memory laid out as the 128-byte-swizzled TMA box (16-byte chunk
+    // c of row r at chunk c ^ (r & 7)); lane 0 stores it.  The box is
+    // rewritten only after the previous bulk group has finished reading it.
+    const int q = warp & 3, h = (warp - 2) >> 2;
+    uint8_t* box = sm + L.box + (size_t)(warp - 2) * kGBox;
+    const uint64_t pol = policy_evict_first();
+    bool pending = false;
+    int tt = 0;
+    bool ok = true;
+    float usum[4][32];
+    for (int i = 0; i < my_units && ok; ++i) {
+      const int4 u = p.units[pair + i * npairs];
+      const int mt = 2 * u.x + rank, nt = u.y;
+      const int row0 = mt * kGM + q * 32;              // first class of this warp's rows
+      const bool rows_exist = row0 < p.m_limit;        // warp-uniform
+      const int n0 = nt * kGN + h * 128;               // first feature of this warp's columns
+#pragma unroll
+      for (int ch = 0; ch < 4; ++ch)
+#pragma unroll
+        for (int c = 0; c < 32; ++c) usum[ch][c] = 0.f;
+      for (int j = 0; j < u.w; ++j, ++tt) {
+        const int b = u.z + j;
+        const int acc = tt & 1;
+        if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[acc], (tt / 2) & 1, p.status))) { ok = false; break; }
+        tc_fence_after();
+        const float sc = p.scale[b];
+        const uint32_t t_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kGN + h * 128);
+#pragma unroll
+        for (int ch = 0; ch < 4; ++ch) {
+          if (rows_exist) {
+            if (lane == 0 && pending) bulk_wait_read0();
+            __syncwarp();
+          }
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+            uint32_t r[16];
+            tmem_ld16(t_base + ch * 32 + hf * 16, r);
+            tmem_ld_wait();
+            float* g = reinterpret_cast<float*>(r);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+              g[c] = sc * __uint_as_float(r[c]);
+              usum[ch][16 * hf + c] += g[c];
+            }
+            if (rows_exist) stage_half(box, lane, hf, g);
+          }
+          if (rows_exist) {
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              for (int k = 0; k < p.ndest; ++k) {
+                const int dd = p.dest[(int64_t)b * p.ndest + k];
+                if (dd >= 0) tma_store_3d_hint(&tmS, box, n0 + ch * 32, row0, dd, pol);
+              }
+              bulk_commit();
+            }
+            pending = true;
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[acc]);
+      }
+      if (ok && p.u_reduce && rows_exist) {
+        // this run's share of the slot total
+#pragma unroll
+        for (int ch = 0; ch < 4; ++ch) {
+          if (lane == 0 && pending) bulk_wait_read0();
+          __syncwarp();
+          stage_half(box, lane, 0, &usum[ch][0]);
+          stage_half(box, lane, 1, &usum[ch][16]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_reduce_add_3d(&tmU, box, n0 + ch * 32, row0, p.u_slot);
+            bulk_commit();
+          }
+          pending = true;
+        }
+      }
+    }
+    if (lane == 0) bulk_wait_all();      // stores done before the CTA exits
+    __syncwarp();
+    if (!ok) atomicExch(cta_err, 1);
+  }
+  __syncthreads();
+  cluster_sync_all();                    // no multicast or remote arrive is still aimed at this CTA
+  if (warp == 1) {
+    // every MMA of this CTA has completed before its accumulator was drained;
+    // after a failure, wait (bounded) for the last commits before releasing
+    if (*cta_err && lane == 0) {
+      int total = 0;
+      for (int i = 0; i < my_units; ++i) total += p.units[pair + i * npairs].w;
+      for (int a = 0; a < 2 && a < total; ++a) {
+        const int last = ((total - 1 - a) / 2) * 2 + a;
+        mbar_wait(&acc_full[a], (last / 2) & 1, p.status);
+      }
+    }
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kGTmem) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+static size_t grad_smem_bytes() { return 1024 + grad_smem().total; }
+
+int tc_grad_max_pairs() {
+  static int mp = -1;
+  if (mp >= 0) return mp;
+  mp = 0;
+  const size_t smem = grad_smem_bytes();
+  if (cudaFuncSetAttribute(tc_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t q = {};
+  q.gridDim = dim3(2);
+  q.blockDim = dim3(kGThreads);
+  q.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  q.attrs = attr;
+  q.numAttrs = 1;
+  int nc = 0;
+  if (cudaOccupancyMaxActiveClusters(&nc, tc_grad_kernel, &q) != cudaSuccess) return 0;
+  mp = nc;
+  return mp;
+}
+
+cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmS, const void* tmU, const TcGradParams& p,
+                           int npairs, cudaStream_t st) {
+  if (p.nunits <= 0) return cudaSuccess;
+  if (npairs < 1) return cudaErrorInvalidValue;
+  const size_t smem = grad_smem_bytes();
+  cudaError_t e = cudaFuncSetAttribute(tc_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int pairs = npairs < p.nunits ? npairs : p.nunits;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(2 * pairs));
+  cfg.blockDim = dim3(kGThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = p.pdl ? 2 : 1;
+  CUtensorMap a, b, o, u;
+  std::memcpy(&a, tmR, sizeof(CUtensorMap));
+  std::memcpy(&b, tmX, sizeof(CUtensorMap));
+  std::memcpy(&o, tmS, sizeof(CUtensorMap));
+  std::memcpy(&u, tmU, sizeof(CUtensorMap));
+  return cudaLaunchKernelEx(&cfg, tc_grad_kernel, a, b, o, u, p);
+}
+
+}  // namespace pgc
