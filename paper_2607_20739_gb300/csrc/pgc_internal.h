@@ -201,9 +201,9 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
 
 // ---- tensor-core gradient contraction (tc_grad.cu) -------------------------
 // G_e = scale_e R_e^T X_e for the runs of partitions in `units`
-// ({class pair tile mp, feature tile nt, first batch, batches}), written as
-// 32 x 32 fp32 boxes into the stores [slot][K][ld] (3-D map) at every dest of
-// the batch; with u_reduce each run's sum is also added (TMA reduce-add) into
+// ({class pair tile mp, feature tile nt, first batch, batches}), written into
+// the stores [slot][K][ld] at every dest of the batch; with u_reduce each
+// run's sum is also added (TMA reduce-add, fp32 box 32 x 32 x 1) into
 // U [c][K][ld] at u_slot.  R is read as MN-major A (box 64 x 64), X as
 // MN-major B (box 64 x 64).
 struct TcGradParams {
@@ -215,7 +215,10 @@ struct TcGradParams {
   const float* scale;       // [nbatch] 1/m_e
   const int32_t* dest;      // [nbatch * ndest] store index or -1
   int ndest;
-  int m_limit;              // classes that exist (K); boxes past it are skipped
+  float* store;             // [slots][K][ld]
+  int64_t ld;               // row pitch of a store (floats)
+  int64_t P;                // K * ld: one store slot
+  int m_limit;              // classes that exist (K); rows past it are not written
   int u_reduce;
   int u_slot;
   int* status;
@@ -224,8 +227,8 @@ struct TcGradParams {
 constexpr int kTcGradMaxRun = 8;   // partitions per unit at most
 // Clusters of two that fit at once (0: the kernel cannot be launched).
 int tc_grad_max_pairs();
-cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmS, const void* tmU, const TcGradParams& p,
-                           int npairs, cudaStream_t st);
+cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, const TcGradParams& p, int npairs,
+                           cudaStream_t st);
 
 // ---- tensor-core logits GEMM with the softmax residual in its epilogue ------
 // (tc_softmax.cu) for every 128-row tile {first X row, first R row, valid

@@ -13,11 +13,13 @@
 // multicast into both CTAs, into a 4-stage ring (2-D TMA, 128-byte swizzle);
 // warp 1 issues tcgen05.mma (M = 128 classes, N = 256 features, K = 16 rows)
 // into one of two TMEM accumulators.  Eight epilogue warps (two per TMEM lane
-// quarter, 128 columns each) drain the other: the scaled gradient goes out as
-// 32 x 32 fp32 boxes with TMA stores (evict-first: the stores are only read
-// back for stragglers), and each thread keeps its row's share of the run's
-// sum in registers, added into U[o_t] with one TMA reduce-add per box at the
-// end of the run.  So U costs one reduce per run instead of one per partition.
+// quarter, 128 columns each) drain the other, 32 x 32 blocks at a time: a
+// block is written row-per-lane into the warp's swizzled scratch, read back
+// transposed and stored as whole 128-byte rows (st.global, evict-first: the
+// stores are only read back for stragglers), so no store waits on another;
+// each thread also keeps its row's share of the run's sum in registers, added
+// into U[o_t] with one TMA reduce-add per block at the end of the run.  So U
+// costs one reduce per run instead of one per partition.
 // Every wait is bounded; the TMEM allocation is released on every path.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -47,15 +49,19 @@ __host__ __device__ constexpr GradSmem grad_smem() {
                   kGS * (kGA + kGB) + kGEpi * kGBox + 16 * 8};
 }
 
+__device__ __forceinline__ void st_global_v4_hint(float* dst, float4 v, uint64_t pol) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(dst), "f"(v.x),
+               "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
+               : "memory");
+}
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 
-// stage 16 values (columns 16 half .. 16 half + 15) of this lane's row into
-// its 128-byte row of a swizzled box (16-byte chunk c at c ^ (row & 7))
-__device__ __forceinline__ void stage_half(uint8_t* box, int lane, int half, const float* v) {
+// stage 8 values (columns 8 qt .. 8 qt + 7) of this lane's row into its
+// 128-byte row of a swizzled box (16-byte chunk c at c ^ (row & 7))
+__device__ __forceinline__ void stage_quarter(uint8_t* box, int lane, int qt, const float* v) {
   float4* rowp = reinterpret_cast<float4*>(box + lane * 128);
-#pragma unroll
-  for (int c = 0; c < 4; ++c)
-    rowp[(4 * half + c) ^ (lane & 7)] = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+  rowp[(2 * qt) ^ (lane & 7)] = make_float4(v[0], v[1], v[2], v[3]);
+  rowp[(2 * qt + 1) ^ (lane & 7)] = make_float4(v[4], v[5], v[6], v[7]);
 }
 
 }  // namespace
@@ -65,7 +71,7 @@ __device__ __forceinline__ void stage_half(uint8_t* box, int lane, int half, con
 // the slot total in them and reads TMEM 16 columns at a time.
 __global__ void __launch_bounds__(kGThreads, 1)
 tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmX,
-               const __grid_constant__ CUtensorMap tmS, const __grid_constant__ CUtensorMap tmU, TcGradParams p) {
+               const __grid_constant__ CUtensorMap tmU, TcGradParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr GradSmem L = grad_smem();
@@ -181,7 +187,6 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
     // rewritten only after the previous bulk group has finished reading it.
     const int q = warp & 3, h = (warp - 2) >> 2;
     uint8_t* box = sm + L.box + (size_t)(warp - 2) * kGBox;
-    const uint64_t pol = policy_evict_first();
     bool pending = false;
     int tt = 0;
     bool ok = true;
@@ -203,36 +208,45 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
         tc_fence_after();
         const float sc = p.scale[b];
         const uint32_t t_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kGN + h * 128);
+        const int32_t* dl = p.dest + (int64_t)b * p.ndest;
 #pragma unroll
         for (int ch = 0; ch < 4; ++ch) {
-          if (rows_exist) {
-            if (lane == 0 && pending) bulk_wait_read0();
+          if (rows_exist && pending) {             // the last U reduce-add has read the box
+            if (lane == 0) bulk_wait_read0();
             __syncwarp();
+            pending = false;
           }
 #pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {
-            uint32_t r[16];
-            tmem_ld16(t_base + ch * 32 + hf * 16, r);
+          for (int qt = 0; qt < 4; ++qt) {
+            uint32_t r[8];
+            tmem_ld8(t_base + ch * 32 + qt * 8, r);
             tmem_ld_wait();
             float* g = reinterpret_cast<float*>(r);
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
+            for (int c = 0; c < 8; ++c) {
               g[c] = sc * __uint_as_float(r[c]);
-              usum[ch][16 * hf + c] += g[c];
+              usum[ch][8 * qt + c] += g[c];
             }
-            if (rows_exist) stage_half(box, lane, hf, g);
+            if (rows_exist) stage_quarter(box, lane, qt, g);
           }
           if (rows_exist) {
-            fence_proxy_async_smem();
+            // read the box back transposed (lane: 16-byte chunk lane % 8 of
+            // rows 4 it + lane / 8) and write whole 128-byte rows
             __syncwarp();
-            if (lane == 0) {
-              for (int k = 0; k < p.ndest; ++k) {
-                const int dd = p.dest[(int64_t)b * p.ndest + k];
-                if (dd >= 0) tma_store_3d_hint(&tmS, box, n0 + ch * 32, row0, dd, pol);
+            const uint64_t pol = policy_evict_first();
+            const int cc = lane & 7;
+            for (int k = 0; k < p.ndest; ++k) {
+              const int dd = dl[k];
+              if (dd < 0) continue;
+              float* dst = p.store + (int64_t)dd * p.P + (int64_t)row0 * p.ld + n0 + ch * 32 + cc * 4;
+#pragma unroll 4
+              for (int it = 0; it < 8; ++it) {
+                const int rr = 4 * it + (lane >> 3);
+                const float4 v = reinterpret_cast<const float4*>(box + rr * 128)[cc ^ (rr & 7)];
+                if (row0 + rr < p.m_limit) st_global_v4_hint(dst + (int64_t)rr * p.ld, v, pol);
               }
-              bulk_commit();
             }
-            pending = true;
+            __syncwarp();
           }
         }
         tc_fence_before();
@@ -245,12 +259,12 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
         for (int ch = 0; ch < 4; ++ch) {
           if (lane == 0 && pending) bulk_wait_read0();
           __syncwarp();
-          stage_half(box, lane, 0, &usum[ch][0]);
-          stage_half(box, lane, 1, &usum[ch][16]);
+#pragma unroll
+          for (int qt = 0; qt < 4; ++qt) stage_quarter(box, lane, qt, &usum[ch][8 * qt]);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_reduce_add_3d(&tmU, box, n0 + ch * 32, row0, p.u_slot);
+            tma_reduce_add_3d_hint(&tmU, box, n0 + ch * 32, row0, p.u_slot, policy_evict_last());
             bulk_commit();
           }
           pending = true;
@@ -309,8 +323,8 @@ int tc_grad_max_pairs() {
   return mp;
 }
 
-cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmS, const void* tmU, const TcGradParams& p,
-                           int npairs, cudaStream_t st) {
+cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, const TcGradParams& p, int npairs,
+                           cudaStream_t st) {
   if (p.nunits <= 0) return cudaSuccess;
   if (npairs < 1) return cudaErrorInvalidValue;
   const size_t smem = grad_smem_bytes();
@@ -331,12 +345,11 @@ cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmS, co
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.pdl ? 2 : 1;
-  CUtensorMap a, b, o, u;
+  CUtensorMap a, b, u;
   std::memcpy(&a, tmR, sizeof(CUtensorMap));
   std::memcpy(&b, tmX, sizeof(CUtensorMap));
-  std::memcpy(&o, tmS, sizeof(CUtensorMap));
   std::memcpy(&u, tmU, sizeof(CUtensorMap));
-  return cudaLaunchKernelEx(&cfg, tc_grad_kernel, a, b, o, u, p);
+  return cudaLaunchKernelEx(&cfg, tc_grad_kernel, a, b, u, p);
 }
 
 }  // namespace pgc
