@@ -114,11 +114,13 @@ def kernel_label(w: W.Workload, single: bool, dom: int) -> str:
     if tensor_core_path(w):
         nt = -(-w.K // 256)
         if dom == 2:
-            return "tc_gemm_kernel, gradient R^T X (tcgen05, 2-CTA clusters)"
+            return "tc_grad_kernel, gradient R^T X (tcgen05, 2-CTA clusters, runs of partitions)"
         if nt in (1, 2, 4, 8):
             return f"tc_logits_softmax_kernel, logits X W^T + softmax residual (tcgen05, {nt}-CTA clusters)"
         return "tc_gemm_kernel, logits X W^T (tcgen05, 2-CTA clusters)"
     if w.loss == "softmax" and w.dtype == "bf16" and w.K <= 16:
+        if -(-w.d // 128) * 128 <= 3072:
+            return "softmax_rows_kernel (whole 16-row tiles per CTA, one pass over X)"
         return "softmax_smallk_kernel (8-CTA clusters, one pass over X)"
     if w.loss == "softmax":
         return "CUDA-core softmax gradient kernels"

@@ -161,6 +161,14 @@ int pgc_destroy(pgc_ctx *ctx);
 /* pgc_strerror — static text for a status code. */
 const char *pgc_strerror(int32_t code);
 
+/* pgc_gradient_path — static name of the kernel path the context computes
+ * per-partition gradients with (fixed at pgc_create): "grad_rows" (logistic,
+ * least squares), "tc_fused" (softmax on the tensor cores, residual in the
+ * logits GEMM), "tc" (tensor cores, separate residual kernel),
+ * "softmax_rows" (few classes, whole rows per CTA), "softmax_cluster" (few
+ * classes, 8-CTA clusters), "softmax_cc" (CUDA cores); "" for NULL. */
+const char *pgc_gradient_path(const pgc_ctx *ctx);
+
 /* pgc_last_cuda_error — name of the CUDA runtime error behind the most
  * recent PGC_ECUDA / PGC_ENOMEM returned on the calling thread (for example
  * "cudaErrorLaunchOutOfResources"), or "" if there was none.  Static text. */

@@ -56,6 +56,7 @@ _sig = {
     "pgc_destroy": (C.c_int, [_vp]),
     "pgc_strerror": (C.c_char_p, [_i32]),
     "pgc_last_cuda_error": (C.c_char_p, []),
+    "pgc_gradient_path": (C.c_char_p, [_vp]),
     "pgc_placement": (C.c_int, [_i32, _i32, _i32, C.POINTER(_i32)]),
     "pgc_schedule": (C.c_int, [_i32, _i32, _i32, _i64, C.POINTER(_i32), C.POINTER(_i32)]),
     "pgc_get_store": (C.c_int, [_vp, _i32, _i32, C.POINTER(C.c_float)]),
@@ -233,6 +234,11 @@ class PGC:
             "eval_partition": self._eval.copy(),
             "fr_rep": self._rep.copy() if self.scheme == FR else None,
         }
+
+    @property
+    def gradient_path(self) -> str:
+        """Name of the kernel path chosen for the per-partition gradients."""
+        return lib.pgc_gradient_path(self._h).decode()
 
     def sync(self):
         _check(lib.pgc_sync(self._h), "pgc_sync")

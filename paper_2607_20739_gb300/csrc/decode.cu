@@ -12,7 +12,8 @@
 
 namespace pgc {
 
-// One CTA per (column slice, evaluated partition).
+// One CTA per (column slice, evaluated partition); a thread sums one float4
+// column over the partition's items (in item order), eight loads in flight.
 __global__ void commit_slice_kernel(CommitArgs a, int64_t slice4) {
   grid_dep_launch();
   grid_dep_wait();
@@ -28,15 +29,13 @@ __global__ void commit_slice_kernel(CommitArgs a, int64_t slice4) {
   for (int64_t j = threadIdx.x; j < w4; j += blockDim.x) {
     const int64_t p = c0 + j;
     float4 acc = f4zero();
-    int it = i0;
-    for (; it + 4 <= i1; it += 4) {
-      const float4 v0 = __ldcg(src + (int64_t)(it + 0) * P4 + p);
-      const float4 v1 = __ldcg(src + (int64_t)(it + 1) * P4 + p);
-      const float4 v2 = __ldcg(src + (int64_t)(it + 2) * P4 + p);
-      const float4 v3 = __ldcg(src + (int64_t)(it + 3) * P4 + p);
-      acc = f4add(f4add(f4add(f4add(acc, v0), v1), v2), v3);
+    for (int it = i0; it < i1; it += 8) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = it + u < i1 ? __ldcg(src + (int64_t)(it + u) * P4 + p) : f4zero();
+#pragma unroll
+      for (int u = 0; u < 8; ++u) acc = f4add(acc, v[u]);
     }
-    for (; it < i1; ++it) acc = f4add(acc, __ldcg(src + (int64_t)it * P4 + p));
     acc = make_float4(acc.x * sc, acc.y * sc, acc.z * sc, acc.w * sc);
     for (int k = 0; k < a.ndest; ++k) {
       const int dst = dest[k];
@@ -64,8 +63,9 @@ cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl) {
   if (a.nE <= 0) return cudaSuccess;
   const int64_t P4 = a.P / 4;
   const int threads = 128;
-  // slices of 512 float4 columns per CTA, one grid row per partition
-  const int64_t slice4 = 512;
+  // one float4 column per thread: slices of 128 columns per CTA, one grid row
+  // per partition (the sums are short and latency-bound: many CTAs)
+  const int64_t slice4 = threads;
   const int64_t bx = (P4 + slice4 - 1) / slice4;
   return launch_maybe_pdl(pdl, commit_slice_kernel, dim3((unsigned)bx, (unsigned)a.nE), dim3(threads), st, a, slice4);
 }

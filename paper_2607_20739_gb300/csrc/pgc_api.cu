@@ -43,13 +43,14 @@ struct Phase {
   int tail = 0;                         // fused tail of the gradient kernel
   // tensor-core softmax path: partitions' Z / R rows padded to 64
   std::vector<int64_t> e_zrow0p;
-  std::vector<int32_t> f_prefix, f_nk, f_aoff, f_mvalid, b_prefix, b_nk, b_aoff, b_boff, b_mvalid;
-  // f_mvalid / b_mvalid hold the M tiles of each batch (forward: row tiles; backward: class tiles)
+  std::vector<int32_t> f_prefix, f_nk, f_aoff, f_mvalid, b_nk, b_aoff, b_boff;
+  // f_mvalid: row tiles of each batch (unfused logits GEMM); b_*: K blocks,
+  // R and X row offsets of each batch (gradient contraction)
   std::vector<int64_t> f_outrow0;
   int64_t zpad_total = 0;
   int64_t* d_e_zrow0p = nullptr;
   int32_t *d_f_prefix = nullptr, *d_f_nk = nullptr, *d_f_aoff = nullptr, *d_f_mvalid = nullptr;
-  int32_t *d_b_prefix = nullptr, *d_b_nk = nullptr, *d_b_aoff = nullptr, *d_b_boff = nullptr, *d_b_mvalid = nullptr;
+  int32_t *d_b_nk = nullptr, *d_b_aoff = nullptr, *d_b_boff = nullptr;
   int64_t* d_f_outrow0 = nullptr;
   // fused logits + residual kernel: 128-row tiles {X row, R row, valid rows, e}
   std::vector<int32_t> q_tiles;
@@ -127,7 +128,12 @@ struct pgc_ctx {
   bool tc = false;           // softmax on the tensor cores (bf16 features)
   bool smallk = false;       // few-class softmax: one-pass cluster kernel
   int sk_nper = 0;           // its 64-feature blocks per CTA slice
-  int sk_nc = 0;             // its clusters
+  int sk_nc = 0;             // its clusters (whole-row variant: its CTAs)
+  bool sk_rows = false;      // the whole-row variant (one CTA per SM, 16-row tiles)
+  int sk_slots = 0;          // its tile slots
+  int sk_box = 1;            // its 64-feature blocks per TMA copy
+  bool sk_tail = true;       // its fused commit + decode (PGC_NO_ROWS_TAIL=1: separate kernels)
+  alignas(64) unsigned char tmXr[128];   // X as [ld/64][rows][64] blocks (box 64 x 16 x ld/64)
   alignas(64) unsigned char tmW16[128];  // Wb [16][ld] for the few-class kernel (box 64 x 16)
   int64_t Ktc = 0;           // classes padded to the forward N tile (256)
   uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]
@@ -136,7 +142,6 @@ struct pgc_ctx {
   alignas(64) unsigned char tmR[128];    // R as MN-major A  (box 64 x 64)
   alignas(64) unsigned char tmXm[128];   // X as MN-major B  (box 64 x 64)
   alignas(64) unsigned char tmZo[128];   // Z fp32 output     (box 32 x 32)
-  alignas(64) unsigned char tmSo[128];   // stores [slot][K][ld] fp32 output (box 32 x 32 x 1)
   alignas(64) unsigned char tmUo[128];   // U [c][K][ld] fp32, reduce-add target
   bool tcf = false;          // logits GEMM with the residual fused (no Z in HBM)
   int tcf_nc = 0;            // its clusters of Ktc / 256 CTAs
@@ -252,13 +257,14 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
       ph.e_item0.push_back((int32_t)ph.items.size());
     }
   } else if (ctx->smallk) {
-    // kSmallKRows-row tiles in partition order; cluster c takes [T c / nc, T (c+1) / nc);
-    // one item per cluster and partition it touches
+    // tiles of tr rows in partition order; cluster (whole-row variant: CTA)
+    // c takes [T c / nc, T (c+1) / nc); one item per cluster and partition it touches
+    const int64_t tr = ctx->sk_rows ? kRowsTileRows : kSmallKRows;
     std::vector<int32_t> te;              // partition of each tile
     for (int e = 0; e < nE; ++e)
-      for (int64_t r0 = 0; r0 < ph.e_rows[e]; r0 += kSmallKRows) {
+      for (int64_t r0 = 0; r0 < ph.e_rows[e]; r0 += tr) {
         ph.sk_tiles.push_back((int32_t)(ph.e_row0[e] + r0));
-        ph.sk_tiles.push_back((int32_t)std::min<int64_t>(kSmallKRows, ph.e_rows[e] - r0));
+        ph.sk_tiles.push_back((int32_t)std::min<int64_t>(tr, ph.e_rows[e] - r0));
         ph.sk_tiles.push_back(0);
         ph.sk_tiles.push_back(0);
         te.push_back(e);
@@ -285,7 +291,6 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
       const int NTf = (int)(ctx->Ktc / 256), MTb = (int)(ctx->Ktc / 128), NTb = (int)(ctx->ld / 256);
       int64_t zp = 0;
       ph.f_prefix.push_back(0);
-      ph.b_prefix.push_back(0);
       for (int e = 0; e < nE; ++e) {
         const int64_t m = ph.e_rows[e];
         ph.e_zrow0p.push_back(zp);
@@ -304,8 +309,6 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
         ph.b_nk.push_back((int32_t)((m + 63) / 64));
         ph.b_aoff.push_back((int32_t)zp);
         ph.b_boff.push_back((int32_t)ph.e_row0[e]);
-        ph.b_mvalid.push_back(MTb);
-        ph.b_prefix.push_back(ph.b_prefix.back() + MTb / 2 * NTb);         // pairs of class tiles
         zp += (m + 127) / 128 * 128;   // whole forward tiles: their TMA stores stay inside the partition
       }
       ph.zpad_total = zp;
@@ -376,6 +379,14 @@ int copy_out(pgc_ctx* ctx, float* dst, const float* src, int on_device) {
 }  // namespace
 
 extern "C" {
+
+const char* pgc_gradient_path(const pgc_ctx* ctx) {
+  if (!ctx) return "";
+  if (ctx->loss != PGC_SOFTMAX) return "grad_rows";
+  if (ctx->tc) return ctx->tcf ? "tc_fused" : "tc";
+  if (ctx->smallk) return ctx->sk_rows ? "softmax_rows" : "softmax_cluster";
+  return "softmax_cc";
+}
 
 const char* pgc_last_cuda_error(void) {
   return g_last_cuda_error == cudaSuccess ? "" : cudaGetErrorName(g_last_cuda_error);
@@ -473,7 +484,36 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
       ctx->tcf = ctx->tcf_nc > 0;
     }
     const char* env2 = std::getenv("PGC_NO_SMALLK");
-    if (!ctx->tc && dtype == PGC_BF16 && !(env2 && env2[0] == '1') && smallk_fits(K, ctx->ld)) {
+    const char* env4 = std::getenv("PGC_NO_ROWS");
+    if (!ctx->tc && dtype == PGC_BF16 && !(env2 && env2[0] == '1') && !(env4 && env4[0] == '1') && K <= 16) {
+      // few classes, rows short enough to hold 16 whole rows per slot: one
+      // CTA per SM, no exchange between CTAs (PGC_NO_ROWS=1 keeps the
+      // cluster kernel)
+      const int64_t ldr = (int64_t)align_up((size_t)d, 128);
+      const int slots = rows_slots(ldr);
+      // TMA copies of up to 8 blocks (16 KB); PGC_ROWS_BOX sets the blocks per copy
+      int box = 1;
+      for (int b = 8; b >= 1; --b)
+        if ((ldr / 64) % b == 0) { box = b; break; }
+      if (const char* env = std::getenv("PGC_ROWS_BOX")) {
+        const int b = std::atoi(env);
+        if (b >= 1 && (ldr / 64) % b == 0) box = b;
+      }
+      ctx->sk_box = box;
+      if (const char* env = std::getenv("PGC_NO_ROWS_TAIL")) ctx->sk_tail = env[0] != '1';
+      // the occupancy query first: it makes the runtime's context current,
+      // which the tensor-map encoder (a driver call) needs
+      const int nctas = slots >= 2 ? rows_max_ctas(ldr, slots) : 0;
+      if (nctas > 0 && make_tmap_bf16_rows(nullptr, nullptr, (uint64_t)ldr, 1024, kRowsTileRows, (uint32_t)box)) {
+        {
+          ctx->ld = ldr;
+          ctx->sk_rows = ctx->smallk = true;
+          ctx->sk_slots = slots;
+          ctx->sk_nc = nctas;
+        }
+      }
+    }
+    if (!ctx->tc && !ctx->smallk && dtype == PGC_BF16 && !(env2 && env2[0] == '1') && smallk_fits(K, ctx->ld)) {
       ctx->sk_nper = (int)((ctx->ld / 64 + 7) / 8);
       ctx->sk_nc = smallk_max_clusters(ctx->sk_nper);
       ctx->smallk = ctx->sk_nc > 0;
@@ -517,7 +557,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   std::vector<uint8_t> tab;
   size_t off = 0;
   std::vector<size_t> offs;
-  constexpr int kTabs = 21;
+  constexpr int kTabs = 19;
   for (auto& ph : ctx->phases) {
     offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
@@ -532,11 +572,9 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     offs.push_back(align_up(off, 16)); put(tab, off, ph.f_aoff);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.f_mvalid);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.f_outrow0);
-    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_prefix);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_nk);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_aoff);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.b_boff);
-    offs.push_back(align_up(off, 16)); put(tab, off, ph.b_mvalid);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.sk_tiles);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.q_tiles);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.g_units);
@@ -627,18 +665,20 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     ph.d_f_aoff = reinterpret_cast<int32_t*>(base + o[10]);
     ph.d_f_mvalid = reinterpret_cast<int32_t*>(base + o[11]);
     ph.d_f_outrow0 = reinterpret_cast<int64_t*>(base + o[12]);
-    ph.d_b_prefix = reinterpret_cast<int32_t*>(base + o[13]);
-    ph.d_b_nk = reinterpret_cast<int32_t*>(base + o[14]);
-    ph.d_b_aoff = reinterpret_cast<int32_t*>(base + o[15]);
-    ph.d_b_boff = reinterpret_cast<int32_t*>(base + o[16]);
-    ph.d_b_mvalid = reinterpret_cast<int32_t*>(base + o[17]);
-    ph.d_sk_tiles = reinterpret_cast<int32_t*>(base + o[18]);
-    ph.d_q_tiles = reinterpret_cast<int32_t*>(base + o[19]);
-    ph.d_g_units = reinterpret_cast<int32_t*>(base + o[20]);
+    ph.d_b_nk = reinterpret_cast<int32_t*>(base + o[13]);
+    ph.d_b_aoff = reinterpret_cast<int32_t*>(base + o[14]);
+    ph.d_b_boff = reinterpret_cast<int32_t*>(base + o[15]);
+    ph.d_sk_tiles = reinterpret_cast<int32_t*>(base + o[16]);
+    ph.d_q_tiles = reinterpret_cast<int32_t*>(base + o[17]);
+    ph.d_g_units = reinterpret_cast<int32_t*>(base + o[18]);
   }
   ctx->loss_desc = nullptr;
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
-  if (ctx->smallk) {
+  if (ctx->sk_rows) {
+    if (!make_tmap_bf16_rows(ctx->tmXr, ctx->X, (uint64_t)ctx->ld, (uint64_t)ctx->total_rows, kRowsTileRows,
+                             (uint32_t)ctx->sk_box))
+      return fail(cudaErrorInvalidValue);
+  } else if (ctx->smallk) {
     const uint64_t pitch = (uint64_t)ctx->ld * 2;
     if (!make_tmap_bf16(ctx->tmXk, ctx->X, ctx->ld, ctx->total_rows, pitch, kSmallKRows) ||
         !make_tmap_bf16(ctx->tmW16, ctx->wb, ctx->ld, 16, pitch, 16))
@@ -651,10 +691,9 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
               make_tmap_bf16(ctx->tmR, ctx->Rb, ctx->Ktc, max_zpad, (uint64_t)ctx->Ktc * 2, 64) &&
               make_tmap_bf16(ctx->tmXm, ctx->X, ctx->ld, ctx->total_rows, pitch, 64);
     const uint64_t zd[2] = {(uint64_t)ctx->Ktc, (uint64_t)max_zpad}, zs[1] = {(uint64_t)ctx->Ktc * 4};
-    const uint64_t sd[3] = {(uint64_t)ctx->ld, (uint64_t)ctx->K, (uint64_t)ctx->owners * ctx->c};
     const uint64_t ud[3] = {(uint64_t)ctx->ld, (uint64_t)ctx->K, (uint64_t)ctx->c};
     const uint64_t ss[2] = {(uint64_t)ctx->ld * 4, (uint64_t)ctx->P * 4};
-    ok = ok && make_tmap_f32_box32(ctx->tmSo, ctx->store, 3, sd, ss) && make_tmap_f32_box32(ctx->tmUo, ctx->U, 3, ud, ss);
+    ok = ok && make_tmap_f32_box32(ctx->tmUo, ctx->U, 3, ud, ss);
     if (ctx->tcf)
       ok = ok && make_tmap_bf16(ctx->tmXq, ctx->X, ctx->ld, ctx->total_rows, pitch, (uint32_t)(128 / (ctx->Ktc / 256))) &&
            make_tmap_bf16(ctx->tmRst, ctx->Rb, ctx->Ktc, max_zpad, (uint64_t)ctx->Ktc * 2, 32);
@@ -757,7 +796,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     // so the backward also forms U[o_t] = sum_e g_e (TMA reduce-add) and the
     // decode reads it instead of re-summing the stores
     const bool u_red = ph.slot >= 0 && ph.ndest == 1;
-    f.a_off = ph.d_f_aoff; f.b_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back(); f.backward = 0;
+    f.a_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back();
     f.out_row0 = ph.d_f_outrow0; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
     if (ctx->tcf) {
       // R straight from the logits GEMM's epilogue
@@ -771,7 +810,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
       PGC_CK(ctx, record_event(ctx));
       PGC_CK(ctx, record_event(ctx));   // empty residual group
     } else {
-      PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, ctx->tmZo, nullptr, f, false, false, ctx->sm_count, st));
+      PGC_CK(ctx, launch_tc_gemm(ctx->tmXk, ctx->tmW, ctx->tmZo, f, ctx->sm_count, st));
       PGC_CK(ctx, record_event(ctx));
       PGC_CK(ctx, launch_softmax_bf16(ctx->Z, ctx->Rb, ctx->Ktc, ctx->K, static_cast<const int32_t*>(ctx->y),
                                       ph.d_e_row0, ph.d_e_rows, ph.d_e_zrow0p, nE, ph.max_rows,
@@ -791,6 +830,22 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     nl[PGC_KRESID] = ctx->tcf ? 0 : 1;
     nl[PGC_KGRADB] = 1;
     need_commit = false;
+  } else if (ctx->sk_rows) {
+    RowsArgs a;
+    a.tiles = reinterpret_cast<const int4*>(ph.d_sk_tiles); a.ntiles = (int)(ph.sk_tiles.size() / 4);
+    a.K = (int)ctx->K; a.y = static_cast<const int32_t*>(ctx->y); a.wb = ctx->wb;
+    a.partials = ctx->partials; a.P = ctx->P; a.ld = ctx->ld; a.nslots = ctx->sk_slots; a.box_blocks = ctx->sk_box;
+    a.status = ctx->status; a.pdl = ctx->pdl ? 1 : 0;
+    if (ctx->sk_tail) {
+      // one kernel per step: commit and decode in the same grid
+      a.tail = 1; a.nE = (int)ph.parts.size(); a.e_item0 = ph.d_e_item0; a.e_scale = ph.d_e_scale;
+      a.e_dest = ph.d_e_dest; a.ndest = ph.ndest; a.store = ctx->store; a.counters = ctx->counters + n;
+      a.dec = dc;
+      need_commit = false;
+      need_decode = false;
+    }
+    nl[PGC_KGRAD] = 1;
+    PGC_CK(ctx, launch_softmax_rows(ctx->tmXr, a, ctx->sk_nc, st));
   } else if (ctx->smallk) {
     SmallKArgs a;
     a.tiles = reinterpret_cast<const int4*>(ph.d_sk_tiles); a.ntiles = (int)(ph.sk_tiles.size() / 4);

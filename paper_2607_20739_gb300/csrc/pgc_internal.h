@@ -155,31 +155,20 @@ struct LossArgs {
 };
 cudaError_t launch_loss(const LossArgs& a, cudaStream_t st);
 
-// ---- tensor-core softmax gradient (tc_gemm.cu) ---------------------------
-// forward  Z[r][k] = sum_j X[r][j] Wb[k][j]   (A = X K-major, B = Wb K-major)
-// backward G_e[k][j] = scale_e sum_r R[r][k] X[r][j]  (A = R MN-major, B = X MN-major)
+// ---- tensor-core logits GEMM (tc_gemm.cu) --------------------------------
+// Z[r][k] = sum_j X[r][j] Wb[k][j] (A = X K-major, B = Wb K-major), for the
+// class counts the fused logits + residual kernel does not cover.
 struct TcGemmParams {
   int nbatch;
   const int* tile_prefix;   // [nbatch + 1] pair tiles before batch b (ceil(MT_b / 2) * NT each)
-  const int* mt_count;      // [nbatch] M tiles (of 128) MT_b
-  int NT;                   // N tiles (of 256) per batch
+  const int* mt_count;      // [nbatch] row tiles (of 128) MT_b
+  int NT;                   // class tiles (of 256) per batch
   const int* nk;            // [nbatch] K blocks (of 64)
-  const int* a_off;         // [nbatch] A row offset (K-major: M rows; MN-major: K rows)
-  const int* b_off;         // [nbatch] B row offset (MN-major: K rows)
+  const int* a_off;         // [nbatch] first X row of the batch
   int total_tiles;
-  int backward;             // 0: forward -> Z rows, 1: backward -> stores
-  // Results leave through TMA stores of 32 x 32 fp32 boxes.  Forward: the
-  // output map is Z [rows][Kpad] (2-D), box at (n, out_row0[b] + m).
-  // Backward: the output map is the stores [slot][K][ld] (3-D), box at
-  // (n, m, dest) for every dest >= 0, scaled by scale[b]; with u_reduce the
-  // same box is also added (TMA reduce-add) into U [c][K][ld] at u_slot.
-  const int64_t* out_row0;  // forward: first Z row of batch b (a multiple of 128)
-  const float* scale;       // backward: 1/m_e
-  const int32_t* dest;      // backward: [nbatch * ndest] store index or -1
-  int ndest;
-  int u_reduce;
-  int u_slot;
-  int m_limit;              // backward: output rows that exist (K); boxes past it are skipped
+  // Results leave through TMA stores of 32 x 32 fp32 boxes into the 2-D map
+  // Z [rows][Kpad], box at (n, out_row0[b] + m).
+  const int64_t* out_row0;  // first Z row of batch b (a multiple of 128)
   int* status;
   int pdl;
 };
@@ -190,8 +179,8 @@ bool make_tmap_bf16(void* tm_out, const void* base, uint64_t inner, uint64_t out
                     uint32_t box_outer);
 // fp32 rank-2 or rank-3 (dims innermost first, byte strides of dims 1..), box {32, 32, 1}
 bool make_tmap_f32_box32(void* tm_out, const void* base, int rank, const uint64_t* dims, const uint64_t* strides);
-cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, const void* tmU, const TcGemmParams& p,
-                           bool a_mn, bool b_mn, int grid, cudaStream_t st);
+cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, const TcGemmParams& p, int grid,
+                           cudaStream_t st);
 // R = softmax(Z) - onehot(y) as bf16, zero for classes K..Kpad-1 and for the
 // rows up to the next multiple of 64; also zeroes zero_buf[0:zero_n] (floats,
 // a multiple of 4) when given.
@@ -276,6 +265,57 @@ bool smallk_fits(int64_t K, int64_t ld);
 int smallk_max_clusters(int nper);
 cudaError_t launch_softmax_smallk(const void* tmX, const void* tmW, const SmallKArgs& a, int nclusters,
                                   cudaStream_t st);
+
+// ---- softmax with few classes, whole rows per CTA (softmax_rows.cu) --------
+// tiles[i] = {first global X row, rows (<= 16), item, flags: 1 first / 2 last
+// tile of a CTA's run in one partition}; CTA c of G takes tiles
+// [ntiles c / G, ntiles (c + 1) / G).  partials[item][K][ld] receives the
+// unscaled gradient sums of the run.
+constexpr int kRowsTileRows = 16;
+constexpr int64_t kRowsMaxLd = 3072;       // the forward keeps a warp's W^T slice in registers
+constexpr int kRowsMaxSlots = 8;
+constexpr int kRowsTmemCols = 512;         // G^T: ld / 128 slices of 16 columns
+constexpr uint32_t kRowsSmemBudget = 227 * 1024 - 9 * 1024;   // the decode plan is static shared memory
+struct RowsArgs {
+  const int4* tiles;
+  int ntiles;
+  int K;
+  const int32_t* y;         // labels per global row
+  const uint16_t* wb;       // bf16 W [16][ld], zero rows past K
+  float* partials;
+  int64_t P;                // K * ld
+  int64_t ld;               // a multiple of 128, at most kRowsMaxLd
+  int nslots;
+  int box_blocks;           // 64-feature blocks per TMA copy (divides ld / 64)
+  int* status;
+  int pdl;
+  // Fused tail (tail = 1): after a grid barrier every CTA commits a share of
+  // the (partition, column) pairs (ordered sum of the partition's items,
+  // times e_scale, into each destination store), then after a second
+  // barrier decodes and updates w (dec) over a share of the columns.  The
+  // grid must be co-resident (one CTA per SM); counters[0..2] are zero
+  // between steps (the last CTA resets them).
+  int tail = 0;
+  int nE = 0;
+  const int32_t* e_item0 = nullptr;  // [nE + 1]
+  const float* e_scale = nullptr;    // [nE]
+  const int32_t* e_dest = nullptr;   // [nE * ndest]
+  int ndest = 1;
+  float* store = nullptr;
+  int* counters = nullptr;
+  DecodeArgs dec;
+};
+// Slots of 16 x ld that fit (0: ld not supported).
+int rows_slots(int64_t ld);
+// CTAs of the grid (one per SM; 0: cannot launch).
+int rows_max_ctas(int64_t ld, int nslots);
+// tmX: X as [ld/64][rows][64] bf16 blocks, box {64, 16, box_blocks} (make_tmap_bf16_rows)
+cudaError_t launch_softmax_rows(const void* tmX, const RowsArgs& a, int nctas, cudaStream_t st);
+// 3-D view of a row-major bf16 [rows][ld] matrix as 64-element blocks: dims
+// {64, rows, ld/64}, box {64, box_rows, box_blocks}, 128-byte swizzle; with
+// tm_out and base both nullptr it only checks that the view can be encoded.
+bool make_tmap_bf16_rows(void* tm_out, const void* base, uint64_t ld, uint64_t rows, uint32_t box_rows,
+                         uint32_t box_blocks);
 
 // ---- misc -------------------------------------------------------------------
 cudaError_t launch_f32_to_bf16(const float* src, uint16_t* dst, int64_t count, cudaStream_t st);

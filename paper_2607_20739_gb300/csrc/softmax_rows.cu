@@ -1,0 +1,477 @@
+// Softmax gradient for few classes (K <= 16, §III with f = log sum_k
+// exp(w_k.x) - w_y.x), bf16 features, one pass over X, whole rows per CTA.
+//
+// For K this small both contractions of the gradient are thin:
+//   Z = X_tile W^T           (16 rows x 16 classes, summed over d)
+//   G += X_tile^T R          (d features x 16 classes, summed over the rows)
+// and the step is bound by reading X once.  Each CTA (one per SM) streams
+// 16-row tiles of whole rows (16 x ld bf16, laid out as 64-feature blocks of
+// 16 rows with 128-byte swizzle by 3-D TMA copies of box_blocks blocks each)
+// through a ring of slots:
+//   1. eight warps form the logits with warp-level mma.sync (m16n8k16, bf16
+//      in, fp32 out), each over its d/8 features, with its slice of W^T held
+//      in registers for the whole step; the eight partial 16 x 16 blocks are
+//      summed through shared memory;
+//   2. one warp forms R = softmax(Z) - onehot(y) (zero past K and past the
+//      partition's rows) in bf16, in the no-swizzle K-major operand layout;
+//   3. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
+//      the 16 rows; A = the resident X tile read MN-major) into a TMEM
+//      accumulator of G^T that spans the CTA's run of tiles in a partition,
+//      and frees the slot with tcgen05.commit.
+// No data leaves the CTA before the end of a run; then four warps write the
+// run's G^T as one partial (one item per CTA and partition).  With the fused
+// tail the same grid then commits (after a grid barrier: every CTA sums a
+// share of the partitions' items in item order, scales by 1/m_e and writes
+// the stores) and decodes (after a second barrier: coefficients from the
+// mask, decode and SGD over a share of the columns); otherwise separate
+// commit and decode kernels follow.
+// Every wait is bounded; the TMEM allocation is released on every path.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <cstring>
+
+#include "tc_common.cuh"
+
+namespace pgc {
+
+namespace {
+
+constexpr int kRR = kRowsTileRows;       // rows per tile (mma.sync M)
+static_assert(kRR == 16, "the forward fragments assume 16-row tiles");
+constexpr int kFw = 8;                   // forward warps (warps 2..9)
+constexpr int kRThreads = 64 + 32 * kFw;
+constexpr int kMaxKs = kRowsMaxLd / 128; // 16-feature steps per forward warp at the largest ld
+constexpr uint32_t kZp = kRR * 16 * 4;   // one warp's partial logits (16 x 16 fp32)
+constexpr uint32_t kRb = kRR * 16 * 2;   // R block (16 rows x 16 classes bf16)
+
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)layout << 61;
+  return d;
+}
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* tm, int x, int y, int z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(
+          smem_u32(dst)),
+      "l"(tm), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& a0, uint32_t& a1, uint32_t& a2, uint32_t& a3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
+// Element (class k, tile row r) of the R block in the K-major layout without
+// swizzle: 8 x 8 core matrices (8 classes x 16 bytes of rows), the core of
+// row chunk r/8 and class group k/8 at (r/8)*256 + (k/8)*128.
+__device__ __forceinline__ uint32_t r_offset(int k, int r) {
+  return (uint32_t)((r >> 3) * 256 + (k >> 3) * 128 + (k & 7) * 16 + (r & 7) * 2);
+}
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Every CTA of the (co-resident) grid arrives on *ctr and waits until all
+// have; bounded.  Called by all threads of the CTA.
+__device__ bool grid_barrier(int* ctr, int* status, int* flag) {
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    atomic_add_acq_rel(ctr, 1);
+    const int target = (int)gridDim.x;
+    if (ld_acquire(ctr) < target) {
+      const uint64_t t0 = globaltimer_ns();
+      for (uint32_t it = 0;; ++it) {
+        if (ld_acquire(ctr) >= target) break;
+        if (it > kWaitMaxIters || ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitMaxNs)) {
+          atomicOr(status, kErrWaitTimeout);
+          ok = 0;
+          break;
+        }
+      }
+    }
+    *flag = ok;
+  }
+  __syncthreads();
+  return *flag != 0;
+}
+
+}  // namespace
+
+struct RowsSmem {
+  uint32_t slot_bytes, zpart, rblk, bars, total;
+};
+__host__ __device__ static RowsSmem rows_smem(int64_t ld, int nslots) {
+  RowsSmem s;
+  s.slot_bytes = (uint32_t)(kRR * ld * 2);
+  s.zpart = (uint32_t)nslots * s.slot_bytes;
+  s.rblk = s.zpart + (uint32_t)nslots * kFw * kZp;
+  s.bars = s.rblk + (uint32_t)nslots * kRb;
+  s.total = s.bars + (3 * kRowsMaxSlots + 4) * 8 + 16;
+  return s;
+}
+
+__global__ void __launch_bounds__(kRThreads, 1)
+softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ RowsArgs a) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ DecodePlan plan;
+  __shared__ int bar_flag;
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int S = a.nslots;
+  const RowsSmem L = rows_smem(a.ld, S);
+  float* zpart = reinterpret_cast<float*>(sm + L.zpart);
+  uint8_t* rblk = sm + L.rblk;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.bars);
+  uint64_t* full = bars;                       // [S] X tile landed
+  uint64_t* empty = bars + kRowsMaxSlots;      // [S] the tile's MMAs are done (slot, R block free)
+  uint64_t* rready = bars + 2 * kRowsMaxSlots; // [S] R block written
+  uint64_t* acc_full = bars + 3 * kRowsMaxSlots;
+  uint64_t* acc_empty = acc_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 2);
+  int* cta_err = reinterpret_cast<int*>(acc_full + 3);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nmt = (int)(a.ld / 128);           // 128-feature M slices of the backward
+  // this CTA's tiles: [T c / G, T (c + 1) / G)
+  const int t0 = (int)((int64_t)a.ntiles * blockIdx.x / gridDim.x);
+  const int t1 = (int)((int64_t)a.ntiles * (blockIdx.x + 1) / gridDim.x);
+  const int n = t1 - t0;
+
+  if (threadIdx.x == 0) {
+    *cta_err = 0;
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+      mbar_init(&rready[s], 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, kFw);
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"((uint32_t)kRowsTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  if (threadIdx.x == 0) grid_dep_launch();
+
+  if (warp == 0 && lane == 0) {
+    // ---- producer: one 3-D copy per tile ------------------------------------
+    bool ok = true;
+    int issued = 0;
+    const uint32_t bytes = L.slot_bytes;
+    const int nkb = (int)(a.ld / 64);
+    // X does not change between steps: no wait for the previous kernel
+    for (int i = 0; i < n && ok; ++i) {
+      const int s = i % S;
+      if (i >= S && !mbar_wait(&empty[s], ((i / S) - 1) & 1, a.status)) { ok = false; break; }
+      mbar_arrive_expect_tx(&full[s], bytes);
+      const int row0 = a.tiles[t0 + i].x;
+      for (int z = 0; z < nkb; z += a.box_blocks)
+        tma_load_3d(sm + (size_t)s * bytes + (size_t)z * (kRR * 128), &tmX, 0, row0, z, &full[s]);
+      ++issued;
+    }
+    if (!ok) atomicExch(cta_err, 1);
+    for (int s = 0; s < S && s < issued; ++s) {
+      const int last = ((issued - 1 - s) / S) * S + s;
+      mbar_wait(&full[s], (last / S) & 1, a.status);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---- backward MMAs: G^T[f][k] += sum_r X[r][f] R[r][k] ----------------------
+    constexpr uint32_t id_bwd = idesc_bf16_f32(128, 16, true, false);
+    bool ok = true;
+    int run = 0;
+    for (int i = 0; i < n && ok; ++i) {
+      const int s = i % S;
+      const int4 tl = a.tiles[t0 + i];
+      const bool first = (tl.w & 1) || i == 0, last = (tl.w & 2) || i == n - 1;
+      if (!mbar_wait(&full[s], (i / S) & 1, a.status) || !mbar_wait(&rready[s], (i / S) & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      if (first && run > 0 && !mbar_wait(acc_empty, (run - 1) & 1, a.status)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t xs = smem_u32(sm + (size_t)s * L.slot_bytes);
+      const uint64_t db = sdesc(smem_u32(rblk + s * kRb), 256, 128, 0);
+      // slice mt: two 64-feature blocks of 16 rows (2 KB apart), 8-row groups
+      // 1 KB apart, at 4 KB steps (the address field counts 16-byte units)
+      const uint64_t da0 = sdesc(xs, 2048, 1024, 2);
+      if (first) {
+        for (int mt = 0; mt < nmt; ++mt) umma_bf16_fresh(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)(mt * 256), db, id_bwd);
+      } else {
+        for (int mt = 0; mt < nmt; ++mt) umma_bf16_acc(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)(mt * 256), db, id_bwd);
+      }
+      umma_commit(&empty[s]);
+      if (last) {
+        umma_commit(acc_full);
+        ++run;
+      }
+    }
+    if (!ok) atomicExch(cta_err, 1);
+  } else if (warp >= 2) {
+    // ---- forward (8 warps), residual (warp 2), run drain (warps 2-5) -------
+    const int fw = warp - 2;
+    const int nks = (int)(a.ld / 128);          // 16-feature steps of this warp
+    const int f0 = fw * nks * 16;               // first feature of this warp
+    const int g = lane >> 2, tq = lane & 3;
+    grid_dep_wait();                            // W is the previous step's update
+    // B fragments of W^T for this warp's features: b0 = W[n][k0 + 2tq ..],
+    // b1 = W[n][k0 + 8 + 2tq ..], n = 8 nb + g
+    uint32_t wf[kMaxKs][2][2];
+#pragma unroll
+    for (int ks = 0; ks < kMaxKs; ++ks)
+#pragma unroll
+      for (int nb = 0; nb < 2; ++nb) {
+        wf[ks][nb][0] = wf[ks][nb][1] = 0u;
+        if (ks < nks) {
+          const uint16_t* wr = a.wb + (int64_t)(8 * nb + g) * a.ld + f0 + ks * 16 + 2 * tq;
+          wf[ks][nb][0] = *reinterpret_cast<const uint32_t*>(wr);
+          wf[ks][nb][1] = *reinterpret_cast<const uint32_t*>(wr + 8);
+        }
+      }
+    // ldmatrix row of this lane: matrix m = lane / 8 (rows 8 (m & 1) .., features 8 (m >> 1) ..)
+    const int lr = ((lane >> 3) & 1) * 8 + (lane & 7), lk = (lane >> 4) * 8;
+    // Every forward warp goes through every tile's named barrier, also after
+    // a failed wait (it then skips its waits and writes), so none is left
+    // waiting at the barrier.
+    bool ok = true;
+    int run = 0;
+    for (int i = 0; i < n; ++i) {
+      const int s = i % S;
+      const int4 tl = a.tiles[t0 + i];
+      const bool last = (tl.w & 2) || i == n - 1;
+      // the residual warp's label, fetched before the tile's work
+      int lab = -1;
+      if (warp == 2 && (lane >> 1) < tl.y) lab = a.y[tl.x + (lane >> 1)];
+      if (ok && !__all_sync(0xffffffffu, mbar_wait(&full[s], (i / S) & 1, a.status))) ok = false;
+      const uint32_t xs = smem_u32(sm + (size_t)s * L.slot_bytes);
+      // four independent accumulator chains (class halves x even / odd steps)
+      float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
+      float d0[4] = {0.f, 0.f, 0.f, 0.f}, d1[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int ks = 0; ks < kMaxKs; ++ks) {
+        if (ks < nks) {
+          const int f = f0 + ks * 16 + lk;
+          const uint32_t ad = xs + (uint32_t)((f >> 6) * 2048 + lr * 128 + ((((f & 63) >> 3) ^ (lr & 7)) << 4));
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(ad, a0, a1, a2, a3);
+          if (ks & 1) {
+            mma16816(d0, a0, a1, a2, a3, wf[ks][0][0], wf[ks][0][1]);
+            mma16816(d1, a0, a1, a2, a3, wf[ks][1][0], wf[ks][1][1]);
+          } else {
+            mma16816(c0, a0, a1, a2, a3, wf[ks][0][0], wf[ks][0][1]);
+            mma16816(c1, a0, a1, a2, a3, wf[ks][1][0], wf[ks][1][1]);
+          }
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        c0[j] += d0[j];
+        c1[j] += d1[j];
+      }
+      // partial logits: rows g, g + 8; classes 2tq, 2tq + 1 (+ 8 for c1)
+      float* zp = zpart + (size_t)(s * kFw + fw) * (kRR * 16);
+      *reinterpret_cast<float2*>(zp + g * 16 + 2 * tq) = make_float2(c0[0], c0[1]);
+      *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 2 * tq) = make_float2(c0[2], c0[3]);
+      *reinterpret_cast<float2*>(zp + g * 16 + 8 + 2 * tq) = make_float2(c1[0], c1[1]);
+      *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 8 + 2 * tq) = make_float2(c1[2], c1[3]);
+      named_sync(1, 32 * kFw);
+      if (warp == 2) {
+        // lane: row lane / 2, classes 8 (lane & 1) .. + 7
+        const int r = lane >> 1, kh = (lane & 1) * 8;
+        float z[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) z[c] = 0.f;
+        const float* zs = zpart + (size_t)s * kFw * (kRR * 16) + r * 16 + kh;
+#pragma unroll
+        for (int w = 0; w < kFw; ++w) {
+          const float4 u0 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16));
+          const float4 u1 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16) + 4);
+          z[0] += u0.x; z[1] += u0.y; z[2] += u0.z; z[3] += u0.w;
+          z[4] += u1.x; z[5] += u1.y; z[6] += u1.z; z[7] += u1.w;
+        }
+        float m = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          if (kh + c < a.K) m = fmaxf(m, z[c]);
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+        float e[8], sum = 0.f;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          e[c] = kh + c < a.K ? expf(z[c] - m) : 0.f;
+          sum += e[c];
+        }
+        sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+        const bool valid = r < tl.y;
+        const float inv = 1.0f / sum;
+        // the MMAs of this slot's previous tile have read its R block
+        if (ok && i >= S && !__all_sync(0xffffffffu, mbar_wait(&empty[s], ((i / S) - 1) & 1, a.status))) ok = false;
+        if (ok) {
+          uint8_t* blk = rblk + s * kRb;
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const int k = kh + c;
+            const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
+            *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, r)) = __float2bfloat16_rn(v);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&rready[s]);
+        }
+      }
+      if (last && ok) {
+        // end of this CTA's run in a partition: G^T slices -> one partial
+        if (!__all_sync(0xffffffffu, mbar_wait(acc_full, run & 1, a.status))) ok = false;
+      }
+      if (last && ok) {
+        // warps w and w + 4 share TMEM lane quarter w % 4 and split the
+        // slices: pairs (2j, 2j + 1) go to the first, then the second, ...
+        tc_fence_after();
+        const int q = warp & 3, half = (warp - 2) >> 2;
+        float* dst = a.partials + (int64_t)tl.z * a.P;
+        for (int mt = 2 * half; mt < nmt; mt += 4) {
+          uint32_t gv[32];
+          tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * 16), gv);   // slices mt, mt + 1
+          tmem_ld_wait();
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            if (mt + h < nmt) {
+              const int f = (mt + h) * 128 + q * 32 + lane;
+#pragma unroll
+              for (int k = 0; k < 16; ++k)
+                if (k < a.K) dst[(int64_t)k * a.ld + f] = __uint_as_float(gv[16 * h + k]);
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty);
+      }
+      if (last) ++run;
+    }
+    if (!ok) atomicExch(cta_err, 1);
+  }
+  __syncthreads();
+  if (a.tail && !*cta_err) {
+    // ---- fused tail: commit, then decode + SGD --------------------------------
+    if (warp == 0) derive_plan_warp(a.dec, plan, lane);   // needs only the mask
+    const int64_t gt = (int64_t)blockIdx.x * blockDim.x + threadIdx.x, GT = (int64_t)gridDim.x * blockDim.x;
+    const int64_t P4 = a.P / 4;
+    bool ok = grid_barrier(a.counters, a.status, &bar_flag);   // every partial is written
+    if (ok) {
+      const float4* src = reinterpret_cast<const float4*>(a.partials);
+      for (int64_t x = gt; x < (int64_t)a.nE * P4; x += GT) {
+        const int e = (int)(x / P4);
+        const int64_t p = x - (int64_t)e * P4;
+        const int i0 = a.e_item0[e], i1 = a.e_item0[e + 1];
+        float4 acc = f4zero();
+        for (int it = i0; it < i1; it += 8) {
+          float4 v[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) v[u] = it + u < i1 ? __ldcg(src + (int64_t)(it + u) * P4 + p) : f4zero();
+#pragma unroll
+          for (int u = 0; u < 8; ++u) acc = f4add(acc, v[u]);
+        }
+        const float sc = a.e_scale[e];
+        acc = make_float4(acc.x * sc, acc.y * sc, acc.z * sc, acc.w * sc);
+        for (int k = 0; k < a.ndest; ++k) {
+          const int dst = a.e_dest[(int64_t)e * a.ndest + k];
+          if (dst >= 0) reinterpret_cast<float4*>(a.store)[(int64_t)dst * P4 + p] = acc;
+        }
+      }
+      ok = grid_barrier(a.counters + 1, a.status, &bar_flag);   // every store is committed
+    }
+    if (ok) {
+      if (blockIdx.x == 0 && warp == 0) write_coeffs_warp(a.dec, lane);
+      decode_columns(a.dec, plan, (int)gt, (int)GT);
+      __syncthreads();
+      // the last CTA out resets the counters for the next step
+      if (threadIdx.x == 0 && atomic_add_acq_rel(a.counters + 2, 1) == (int)gridDim.x - 1) {
+        a.counters[0] = 0;
+        a.counters[1] = 0;
+        a.counters[2] = 0;
+        __threadfence();
+      }
+    }
+  }
+  if (warp == 1) {
+    // after a failure, wait (bounded) for the last commit before releasing TMEM
+    if (*cta_err && lane == 0 && n > 0) {
+      const int s = (n - 1) % S;
+      mbar_wait(&empty[s], ((n - 1) / S) & 1, a.status);
+    }
+    __syncwarp();
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kRowsTmemCols)
+                 : "memory");
+  }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+int rows_slots(int64_t ld) {
+  if (ld % 128 != 0 || ld > kRowsMaxLd) return 0;
+  int s = kRowsMaxSlots;
+  while (s >= 2 && rows_smem(ld, s).total + 1024 > kRowsSmemBudget) --s;
+  return s >= 2 ? s : 0;
+}
+
+static size_t rows_smem_bytes(int64_t ld, int nslots) { return 1024 + rows_smem(ld, nslots).total; }
+
+int rows_max_ctas(int64_t ld, int nslots) {
+  const size_t smem = rows_smem_bytes(ld, nslots);
+  if (cudaFuncSetAttribute(softmax_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+      cudaSuccess)
+    return 0;
+  int per_sm = 0, sms = 0, dev = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, softmax_rows_kernel, kRThreads, smem) != cudaSuccess)
+    return 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                cudaSuccess)
+    return 0;
+  return per_sm >= 1 ? sms : 0;   // one CTA per SM (tensor memory)
+}
+
+cudaError_t launch_softmax_rows(const void* tmX, const RowsArgs& a, int nctas, cudaStream_t st) {
+  if (a.ntiles <= 0) return cudaSuccess;
+  if (nctas < 1 || a.nslots < 2 || a.nslots > kRowsMaxSlots) return cudaErrorInvalidValue;
+  const size_t smem = rows_smem_bytes(a.ld, a.nslots);
+  cudaError_t e = cudaFuncSetAttribute(softmax_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)nctas);
+  cfg.blockDim = dim3(kRThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = a.pdl ? 1 : 0;
+  CUtensorMap x;
+  std::memcpy(&x, tmX, sizeof(CUtensorMap));
+  return cudaLaunchKernelEx(&cfg, softmax_rows_kernel, x, a);
+}
+
+}  // namespace pgc

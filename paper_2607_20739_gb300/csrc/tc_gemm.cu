@@ -1,22 +1,20 @@
-// Tensor-core GEMMs of the softmax gradient (§III with f = log sum_k exp(w_k.x)
-// - w_y.x), on the sm_103a tcgen05 path:
+// Logits GEMM of the tensor-core softmax path (§III with f = log sum_k
+// exp(w_k.x) - w_y.x) for class counts whose 256-class tiles do not form a
+// cluster of 1, 2, 4 or 8 CTAs (the fused kernel covers those):
 //
-//   forward   Z[r][k]   = sum_j X[r][j] W[k][j]                 A = X (K-major),  B = W (K-major)
-//   backward  G_e[k][j] = (1/m_e) sum_{r in D_e} R[r][k] X[r][j]  A = R (MN-major), B = X (MN-major)
+//   Z[r][k] = sum_j X[r][j] W[k][j]       A = X (K-major), B = W (K-major)
 //
-// with R = softmax(Z) - onehot(y) in bf16 between them.  Both are one
+// followed by the residual kernel R = softmax(Z) - onehot(y).  One
 // persistent, warp-specialised kernel launched as clusters of two CTAs: the
-// pair computes the M tiles 2i and 2i+1 of the same (batch, N tile), so the
-// B tile is common; each CTA loads its own 128x64 A tile and one 128-row half
-// of the 256x64 B tile, multicast into both CTAs, into a 4-stage
+// pair computes the row tiles 2i and 2i+1 of the same (batch, class tile), so
+// the B tile is common; each CTA loads its own 128x64 A tile and one 128-row
+// half of the 256x64 B tile, multicast into both CTAs, into a 4-stage
 // shared-memory ring with 2-D TMA (cp.async.bulk.tensor, 128-byte swizzle).
 // A stage is refilled once the MMAs of both CTAs have read it.  Warp 1 issues
 // tcgen05.mma.cta_group::1.kind::f16 (bf16 in, fp32 accumulate) into one of
 // two 128x256 TMEM accumulators, and warps 2-5 drain the other accumulator
 // with tcgen05.ld, stage 32 x 32 fp32 boxes in (swizzled) shared memory and
-// write them with TMA stores (forward: logits; backward: the new gradient
-// straight into every store that keeps it, scaled by 1/m_e, and optionally
-// added into the slot total U[o_t] with a TMA reduce-add).
+// write them to Z with TMA stores.
 // Every wait is bounded; the TMEM allocation is released on every path.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -55,10 +53,9 @@ __device__ __forceinline__ bool decode_tile(const TcGemmParams& p, int t, int ra
   return mt < p.mt_count[b];
 }
 
-template <bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-               const __grid_constant__ CUtensorMap tmOut, const __grid_constant__ CUtensorMap tmU, TcGemmParams p) {
+               const __grid_constant__ CUtensorMap tmOut, TcGemmParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -118,18 +115,8 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         mbar_arrive_expect_tx(&full[s], kABytes + kBBytes);
         uint8_t* a_dst = sA + (size_t)s * kABytes;
         uint8_t* b_dst = sB + (size_t)s * kBBytes;
-        if (!A_MN) {
-          tma_load_2d(a_dst, &tmA, kb * kTK, p.a_off[b] + mt * kTM, &full[s]);
-        } else {
-          for (int j = 0; j < kTM / 64; ++j)
-            tma_load_2d(a_dst + j * 8192, &tmA, mt * kTM + j * 64, p.a_off[b] + kb * kTK, &full[s]);
-        }
-        if (!B_MN) {
-          tma_load_2d_mc(b_dst + rank * (kBBytes / 2), &tmB, kb * kTK, nt * kTN + rank * (kTN / 2), &full[s], kPair);
-        } else {
-          for (int j = 2 * rank; j < 2 * rank + 2; ++j)
-            tma_load_2d_mc(b_dst + j * 8192, &tmB, nt * kTN + j * 64, p.b_off[b] + kb * kTK, &full[s], kPair);
-        }
+        tma_load_2d(a_dst, &tmA, kb * kTK, p.a_off[b] + mt * kTM, &full[s]);
+        tma_load_2d_mc(b_dst + rank * (kBBytes / 2), &tmB, kb * kTK, nt * kTN + rank * (kTN / 2), &full[s], kPair);
       }
     }
     if (!ok) atomicExch(&cta_err, 1);
@@ -140,7 +127,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
     }
   } else if (warp == 1 && lane == 0) {
     // ---- MMA issuer --------------------------------------------------------
-    constexpr uint32_t idesc = idesc_bf16_f32(kTM, kTN, A_MN, B_MN);
+    constexpr uint32_t idesc = idesc_bf16_f32(kTM, kTN, false, false);
     int it = 0;
     bool ok = true;
     for (int i = 0; i < my_tiles && ok; ++i) {
@@ -160,11 +147,9 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
 #pragma unroll
         for (int kk = 0; kk < kTK / 16; ++kk) {
           // K-major: the next 16 K elements are 32 bytes further along each
-          // 128-byte row; MN-major: 16 K rows further, 2 groups of 8 rows.
-          const uint64_t da = A_MN ? smem_desc_sw128(a_base + kk * 2048, 8192, 1024)
-                                   : smem_desc_sw128(a_base + kk * 32, 16, 1024);
-          const uint64_t db = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
-                                   : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+          // 128-byte row
+          const uint64_t da = smem_desc_sw128(a_base + kk * 32, 16, 1024);
+          const uint64_t db = smem_desc_sw128(b_base + kk * 32, 16, 1024);
           umma_bf16(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
         }
         umma_commit_mc(&empty[s], kPair);  // this CTA is done with the stage, in both CTAs' count
@@ -193,8 +178,7 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
       }
       tc_fence_after();
       const int row0 = mt * kTM + q * 32;              // first tile row of this warp
-      const bool rows_exist = real && (!p.backward || row0 < p.m_limit);
-      const float sc = p.backward ? p.scale[b] : 1.0f;
+      const bool rows_exist = real;
       const uint32_t t_base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kTN);
       for (int ch = 0; ch < kTN / 32; ++ch) {
         uint32_t r[32];
@@ -207,21 +191,12 @@ tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ 
         float4* rowp = reinterpret_cast<float4*>(box + lane * 128);
 #pragma unroll
         for (int v = 0; v < 8; ++v)
-          rowp[v ^ (lane & 7)] = make_float4(sc * __uint_as_float(r[4 * v]), sc * __uint_as_float(r[4 * v + 1]),
-                                             sc * __uint_as_float(r[4 * v + 2]), sc * __uint_as_float(r[4 * v + 3]));
+          rowp[v ^ (lane & 7)] = make_float4(__uint_as_float(r[4 * v]), __uint_as_float(r[4 * v + 1]),
+                                             __uint_as_float(r[4 * v + 2]), __uint_as_float(r[4 * v + 3]));
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          const int n0 = nt * kTN + ch * 32;
-          if (!p.backward) {
-            tma_store_2d(&tmOut, box, n0, (int)p.out_row0[b] + row0);
-          } else {
-            for (int k = 0; k < p.ndest; ++k) {
-              const int dd = p.dest[(int64_t)b * p.ndest + k];
-              if (dd >= 0) tma_store_3d(&tmOut, box, n0, row0, dd);
-            }
-            if (p.u_reduce) tma_reduce_add_3d(&tmU, box, n0, row0, p.u_slot);
-          }
+          tma_store_2d(&tmOut, box, nt * kTN + ch * 32, (int)p.out_row0[b] + row0);
           bulk_commit();
         }
         ++nbox;
@@ -283,6 +258,24 @@ bool make_tmap_bf16(void* tm_out, const void* base, uint64_t inner, uint64_t out
   return r == CUDA_SUCCESS;
 }
 
+bool make_tmap_bf16_rows(void* tm_out, const void* base, uint64_t ld, uint64_t rows, uint32_t box_rows,
+                         uint32_t box_blocks) {
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn || ld % 64 != 0 || box_blocks < 1 || box_blocks > 256 || (ld / 64) % box_blocks != 0 || rows == 0)
+    return false;
+  alignas(64) CUtensorMap probe;
+  CUtensorMap* out = tm_out ? reinterpret_cast<CUtensorMap*>(tm_out) : &probe;
+  const void* b = base ? base : reinterpret_cast<const void*>(uintptr_t(1) << 20);
+  cuuint64_t dims[3] = {64, rows, ld / 64};
+  cuuint64_t strides[2] = {ld * 2, 128};
+  cuuint32_t box[3] = {64, box_rows, box_blocks};
+  cuuint32_t estr[3] = {1, 1, 1};
+  const CUresult r = fn(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(b), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 bool make_tmap_f32_box32(void* tm_out, const void* base, int rank, const uint64_t* dims, const uint64_t* strides) {
   PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
   if (!fn || rank < 2 || rank > 3) return false;
@@ -301,10 +294,10 @@ static size_t gemm_smem_bytes() {
   return 1024 + kGStages * (size_t)(kABytes + kBBytes) + kEpiBytes + sizeof(uint64_t) * (2 * kGStages + 4) + 16;
 }
 
-template <bool A_MN, bool B_MN>
-static cudaError_t launch_tc(const void* tmA, const void* tmB, const void* tmOut, const void* tmU,
-                             const TcGemmParams& p, int grid, cudaStream_t st) {
-  auto kern = tc_gemm_kernel<A_MN, B_MN>;
+cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, const TcGemmParams& p, int grid,
+                           cudaStream_t st) {
+  if (p.total_tiles <= 0) return cudaSuccess;
+  auto kern = tc_gemm_kernel;
   const size_t smem = gemm_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -323,8 +316,7 @@ static cudaError_t launch_tc(const void* tmA, const void* tmB, const void* tmOut
   cfg.attrs = attr;
   cfg.numAttrs = p.pdl ? 2 : 1;
   // one pair per two SMs that can hold it at once
-  static int max_pairs[2] = {0, 0};
-  int& mp = max_pairs[A_MN ? 1 : 0];
+  static int mp = 0;
   if (mp == 0) {
     cudaLaunchConfig_t q = cfg;
     q.gridDim = dim3(2);
@@ -338,21 +330,11 @@ static cudaError_t launch_tc(const void* tmA, const void* tmB, const void* tmOut
   if (pairs > p.total_tiles) pairs = p.total_tiles;
   if (pairs < 1) pairs = 1;
   cfg.gridDim = dim3((unsigned)(2 * pairs));
-  CUtensorMap a, b, o, u;
+  CUtensorMap a, b, o;
   std::memcpy(&a, tmA, sizeof(CUtensorMap));
   std::memcpy(&b, tmB, sizeof(CUtensorMap));
   std::memcpy(&o, tmOut, sizeof(CUtensorMap));
-  std::memcpy(&u, tmU ? tmU : tmOut, sizeof(CUtensorMap));
-  return cudaLaunchKernelEx(&cfg, kern, a, b, o, u, p);
-}
-
-cudaError_t launch_tc_gemm(const void* tmA, const void* tmB, const void* tmOut, const void* tmU, const TcGemmParams& p,
-                           bool a_mn, bool b_mn, int grid, cudaStream_t st) {
-  if (p.total_tiles <= 0) return cudaSuccess;
-  if (p.u_reduce && !tmU) return cudaErrorInvalidValue;
-  if (!a_mn && !b_mn) return launch_tc<false, false>(tmA, tmB, tmOut, tmU, p, grid, st);
-  if (a_mn && b_mn) return launch_tc<true, true>(tmA, tmB, tmOut, tmU, p, grid, st);
-  return cudaErrorInvalidValue;
+  return cudaLaunchKernelEx(&cfg, kern, a, b, o, p);
 }
 
 }  // namespace pgc

@@ -239,7 +239,7 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
               const int dd = dl[k];
               if (dd < 0) continue;
               float* dst = p.store + (int64_t)dd * p.P + (int64_t)row0 * p.ld + n0 + ch * 32 + cc * 4;
-#pragma unroll 4
+#pragma unroll 1
               for (int it = 0; it < 8; ++it) {
                 const int rr = 4 * it + (lane >> 3);
                 const float4 v = reinterpret_cast<const float4*>(box + rr * 128)[cc ^ (rr & 7)];

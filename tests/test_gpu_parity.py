@@ -65,6 +65,19 @@ def test_parity_with_oracle(libpgc, cuda, name):
     g.close()
 
 
+@pytest.mark.parametrize("name", ["fr_smallk_k10_unequal_rows", "cr_smallk_k16_d1000"])
+def test_parity_cluster_few_class_kernel(libpgc, cuda, monkeypatch, name):
+    """The few-class cases again with the 8-CTA cluster kernel (the path taken
+    when the whole-row kernel does not apply)."""
+    monkeypatch.setenv("PGC_NO_ROWS", "1")
+    w, T = CASES[name]
+    Xs, ys, masks = generate(w, T)
+    g, grecs = run_gpu(libpgc, w, Xs, ys, masks)
+    orecs = run_oracle(w, Xs, ys, masks)
+    compare_runs(w, grecs, orecs)
+    g.close()
+
+
 def test_stores_hold_the_scheduled_gradients(libpgc, cuda):
     """After each step every worker's store slot l holds the gradient of its
     slot-l partition at the step it was last evaluated (s(t,i,j), §V-B)."""
@@ -149,4 +162,39 @@ def test_teacher_forced_gradient(libpgc, cuda):
         g.step(masks[t], grad)
         rec = o.step(masks[t])
         assert rel_err(grad.reshape(w.K, w.d), rec["grad"]) < 2e-2
+    g.close()
+
+
+EXPECTED_PATHS = {
+    "fr_n4_logistic_d64": "grad_rows",
+    "cr_f32_softmax_k3": "softmax_cc",
+    "fr_bf16_softmax_k2": "softmax_rows",
+    "fr_smallk_k10_unequal_rows": "softmax_rows",
+    "cr_smallk_k16_d1000": "softmax_rows",
+    "cr_tc_k300_d320_m200": "tc_fused",
+    "cr_tc_k2000_nt8": "tc_fused",
+    "fr_tc_k1500_unfused": "tc",
+}
+
+
+@pytest.mark.parametrize("name", list(EXPECTED_PATHS))
+def test_gradient_path_chosen(libpgc, cuda, name):
+    """Each workload shape runs on the kernel path meant for it (a silent
+    fallback to a slower path would still pass parity)."""
+    w, _ = CASES[name]
+    g = libpgc.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr)
+    assert g.gradient_path == EXPECTED_PATHS[name]
+    g.close()
+
+
+def test_gradient_path_overrides(libpgc, cuda, monkeypatch):
+    w, _ = CASES["fr_smallk_k10_unequal_rows"]
+    monkeypatch.setenv("PGC_NO_ROWS", "1")
+    g = libpgc.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr)
+    assert g.gradient_path == "softmax_cluster"
+    g.close()
+    w, _ = CASES["cr_tc_k300_d320_m200"]
+    monkeypatch.setenv("PGC_NO_FUSED", "1")
+    g = libpgc.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr)
+    assert g.gradient_path == "tc"
     g.close()
