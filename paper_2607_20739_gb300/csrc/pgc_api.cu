@@ -129,11 +129,11 @@ struct pgc_ctx {
   bool smallk = false;       // few-class softmax: one-pass cluster kernel
   int sk_nper = 0;           // its 64-feature blocks per CTA slice
   int sk_nc = 0;             // its clusters (whole-row variant: its CTAs)
-  bool sk_rows = false;      // the whole-row variant (one CTA per SM, 16-row tiles)
+  bool sk_rows = false;      // the whole-row variant (one CTA per SM, kRowsTileRows-row tiles)
   int sk_slots = 0;          // its tile slots
   int sk_box = 1;            // its 64-feature blocks per TMA copy
   bool sk_tail = true;       // its fused commit + decode (PGC_NO_ROWS_TAIL=1: separate kernels)
-  alignas(64) unsigned char tmXr[128];   // X as [ld/64][rows][64] blocks (box 64 x 16 x ld/64)
+  alignas(64) unsigned char tmXr[128];   // X as [ld/64][rows][64] blocks (box 64 x kRowsTileRows x sk_box)
   alignas(64) unsigned char tmW16[128];  // Wb [16][ld] for the few-class kernel (box 64 x 16)
   int64_t Ktc = 0;           // classes padded to the forward N tile (256)
   uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]

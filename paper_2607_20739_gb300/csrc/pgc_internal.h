@@ -267,7 +267,7 @@ cudaError_t launch_softmax_smallk(const void* tmX, const void* tmW, const SmallK
                                   cudaStream_t st);
 
 // ---- softmax with few classes, whole rows per CTA (softmax_rows.cu) --------
-// tiles[i] = {first global X row, rows (<= 16), item, flags: 1 first / 2 last
+// tiles[i] = {first global X row, rows (<= kRowsTileRows), item, flags: 1 first / 2 last
 // tile of a CTA's run in one partition}; CTA c of G takes tiles
 // [ntiles c / G, ntiles (c + 1) / G).  partials[item][K][ld] receives the
 // unscaled gradient sums of the run.
@@ -305,11 +305,11 @@ struct RowsArgs {
   int* counters = nullptr;
   DecodeArgs dec;
 };
-// Slots of 16 x ld that fit (0: ld not supported).
+// Slots of kRowsTileRows x ld that fit (0: ld not supported).
 int rows_slots(int64_t ld);
 // CTAs of the grid (one per SM; 0: cannot launch).
 int rows_max_ctas(int64_t ld, int nslots);
-// tmX: X as [ld/64][rows][64] bf16 blocks, box {64, 16, box_blocks} (make_tmap_bf16_rows)
+// tmX: X as [ld/64][rows][64] bf16 blocks, box {64, kRowsTileRows, box_blocks} (make_tmap_bf16_rows)
 cudaError_t launch_softmax_rows(const void* tmX, const RowsArgs& a, int nctas, cudaStream_t st);
 // 3-D view of a row-major bf16 [rows][ld] matrix as 64-element blocks: dims
 // {64, rows, ld/64}, box {64, box_rows, box_blocks}, 128-byte swizzle; with

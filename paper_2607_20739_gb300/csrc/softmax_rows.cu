@@ -5,15 +5,18 @@
 //   Z = X_tile W^T           (16 rows x 16 classes, summed over d)
 //   G += X_tile^T R          (d features x 16 classes, summed over the rows)
 // and the step is bound by reading X once.  Each CTA (one per SM) streams
-// 16-row tiles of whole rows (16 x ld bf16, laid out as 64-feature blocks of
-// 16 rows with 128-byte swizzle by 3-D TMA copies of box_blocks blocks each)
-// through a ring of slots:
+// tiles of kRR whole rows (kRR x ld bf16, laid out as 64-feature blocks of kRR
+// rows with 128-byte swizzle by 3-D TMA copies of box_blocks blocks each)
+// through a ring of slots; 8-row tiles keep four 48 KB slots in flight at
+// d = 3072 (the MMA shapes stay at 16 rows: the extra rows repeat the tile's
+// and carry zero residuals):
 //   1. eight warps form the logits with warp-level mma.sync (m16n8k16, bf16
 //      in, fp32 out), each over its d/8 features, with its slice of W^T held
 //      in registers for the whole step; the eight partial 16 x 16 blocks are
 //      summed through shared memory;
-//   2. one warp forms R = softmax(Z) - onehot(y) (zero past K and past the
-//      partition's rows) in bf16, in the no-swizzle K-major operand layout;
+//   2. a warp of its own forms R = softmax(Z) - onehot(y) (zero past K and
+//      past the partition's rows) in bf16, in the no-swizzle K-major operand
+//      layout, while the eight go on with the next tile;
 //   3. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
 //      the 16 rows; A = the resident X tile read MN-major) into a TMEM
 //      accumulator of G^T that spans the CTA's run of tiles in a partition,
@@ -37,13 +40,15 @@ namespace pgc {
 
 namespace {
 
-constexpr int kRR = kRowsTileRows;       // rows per tile (mma.sync M)
-static_assert(kRR == 16, "the forward fragments assume 16-row tiles");
+constexpr int kRR = kRowsTileRows;       // rows per tile
+static_assert(kRR == 8 || kRR == 16, "tiles of 8 or 16 rows (mma.sync M = 16, tcgen05 K = 16)");
+constexpr uint32_t kBlk = kRR * 128;      // one 64-feature block of the tile
 constexpr int kFw = 8;                   // forward warps (warps 2..9)
-constexpr int kRThreads = 64 + 32 * kFw;
+constexpr int kRWarp = 2 + kFw;          // the residual warp
+constexpr int kRThreads = 64 + 32 * kFw + 32;
 constexpr int kMaxKs = kRowsMaxLd / 128; // 16-feature steps per forward warp at the largest ld
-constexpr uint32_t kZp = kRR * 16 * 4;   // one warp's partial logits (16 x 16 fp32)
-constexpr uint32_t kRb = kRR * 16 * 2;   // R block (16 rows x 16 classes bf16)
+constexpr uint32_t kZp = kRR * 16 * 4;   // one warp's partial logits (kRR rows x 16 classes fp32)
+constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16; rows past kRR stay zero)
 
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
   uint64_t d = 0;
@@ -73,7 +78,6 @@ __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
-__device__ __forceinline__ void named_sync(int id, int n) { asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory"); }
 // Element (class k, tile row r) of the R block in the K-major layout without
 // swizzle: 8 x 8 core matrices (8 classes x 16 bytes of rows), the core of
 // row chunk r/8 and class group k/8 at (r/8)*256 + (k/8)*128.
@@ -122,7 +126,7 @@ __host__ __device__ static RowsSmem rows_smem(int64_t ld, int nslots) {
   s.zpart = (uint32_t)nslots * s.slot_bytes;
   s.rblk = s.zpart + (uint32_t)nslots * kFw * kZp;
   s.bars = s.rblk + (uint32_t)nslots * kRb;
-  s.total = s.bars + (3 * kRowsMaxSlots + 4) * 8 + 16;
+  s.total = s.bars + (4 * kRowsMaxSlots + 4) * 8 + 16;
   return s;
 }
 
@@ -140,7 +144,8 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
   uint64_t* full = bars;                       // [S] X tile landed
   uint64_t* empty = bars + kRowsMaxSlots;      // [S] the tile's MMAs are done (slot, R block free)
   uint64_t* rready = bars + 2 * kRowsMaxSlots; // [S] R block written
-  uint64_t* acc_full = bars + 3 * kRowsMaxSlots;
+  uint64_t* zready = bars + 3 * kRowsMaxSlots; // [S] every forward warp's partial logits written
+  uint64_t* acc_full = bars + 4 * kRowsMaxSlots;
   uint64_t* acc_empty = acc_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 2);
   int* cta_err = reinterpret_cast<int*>(acc_full + 3);
@@ -158,11 +163,16 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
       mbar_init(&rready[s], 1);
+      mbar_init(&zready[s], kFw);
     }
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, kFw);
     fence_mbar_init();
   }
+  // R blocks start zeroed: with 8-row tiles their rows 8-15 stay zero
+  for (uint32_t k = threadIdx.x; k < (uint32_t)S * kRb / 16; k += blockDim.x)
+    reinterpret_cast<uint4*>(rblk)[k] = make_uint4(0u, 0u, 0u, 0u);
+  fence_proxy_async_smem();
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"((uint32_t)kRowsTmemCols)
@@ -188,7 +198,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       mbar_arrive_expect_tx(&full[s], bytes);
       const int row0 = a.tiles[t0 + i].x;
       for (int z = 0; z < nkb; z += a.box_blocks)
-        tma_load_3d(sm + (size_t)s * bytes + (size_t)z * (kRR * 128), &tmX, 0, row0, z, &full[s]);
+        tma_load_3d(sm + (size_t)s * bytes + (size_t)z * kBlk, &tmX, 0, row0, z, &full[s]);
       ++issued;
     }
     if (!ok) atomicExch(cta_err, 1);
@@ -213,13 +223,16 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       tc_fence_after();
       const uint32_t xs = smem_u32(sm + (size_t)s * L.slot_bytes);
       const uint64_t db = sdesc(smem_u32(rblk + s * kRb), 256, 128, 0);
-      // slice mt: two 64-feature blocks of 16 rows (2 KB apart), 8-row groups
-      // 1 KB apart, at 4 KB steps (the address field counts 16-byte units)
-      const uint64_t da0 = sdesc(xs, 2048, 1024, 2);
+      // slice mt: two 64-feature blocks kBlk apart; the K = 16 rows of one
+      // MMA are two 8-row groups 1 KB apart (16-row tiles) or the tile's 8
+      // rows twice (8-row tiles: R's rows 8-15 are zero); slices 2 kBlk
+      // apart (the address field counts 16-byte units)
+      const uint64_t da0 = sdesc(xs, kBlk, kRR == 16 ? 1024 : 0, 2);
+      constexpr uint64_t kStep = (2 * kBlk) >> 4;
       if (first) {
-        for (int mt = 0; mt < nmt; ++mt) umma_bf16_fresh(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)(mt * 256), db, id_bwd);
+        for (int mt = 0; mt < nmt; ++mt) umma_bf16_fresh(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)mt * kStep, db, id_bwd);
       } else {
-        for (int mt = 0; mt < nmt; ++mt) umma_bf16_acc(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)(mt * 256), db, id_bwd);
+        for (int mt = 0; mt < nmt; ++mt) umma_bf16_acc(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)mt * kStep, db, id_bwd);
       }
       umma_commit(&empty[s]);
       if (last) {
@@ -228,8 +241,60 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       }
     }
     if (!ok) atomicExch(cta_err, 1);
+  } else if (warp == kRWarp) {
+    // ---- residual: R = softmax(Z) - onehot(y) per tile --------------------
+    // lane: row lane / 2 (rows past kRR: idle lanes), classes 8 (lane & 1) .. + 7.
+    // zpart[s] and the R block of slot s are free again once the tile's slot
+    // was refilled (its full wait implies the previous MMAs completed).
+    const int r = (lane >> 1) & (kRR - 1), kh = (lane & 1) * 8;
+    const bool live = (lane >> 1) < kRR;
+    bool ok = true;
+    for (int i = 0; i < n && ok; ++i) {
+      const int s = i % S;
+      const int4 tl = a.tiles[t0 + i];
+      const bool valid = live && r < tl.y;
+      const int lab = valid ? a.y[tl.x + r] : -1;        // fetched before the wait
+      if (!__all_sync(0xffffffffu, mbar_wait(&zready[s], (i / S) & 1, a.status))) { ok = false; break; }
+      float z[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c) z[c] = 0.f;
+      const float* zs = zpart + (size_t)s * kFw * (kRR * 16) + r * 16 + kh;
+#pragma unroll
+      for (int w = 0; w < kFw; ++w) {
+        const float4 u0 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16));
+        const float4 u1 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16) + 4);
+        z[0] += u0.x; z[1] += u0.y; z[2] += u0.z; z[3] += u0.w;
+        z[4] += u1.x; z[5] += u1.y; z[6] += u1.z; z[7] += u1.w;
+      }
+      float m = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        if (kh + c < a.K) m = fmaxf(m, z[c]);
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+      float e[8], sum = 0.f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        e[c] = kh + c < a.K ? expf(z[c] - m) : 0.f;
+        sum += e[c];
+      }
+      sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+      const float inv = 1.0f / sum;
+      uint8_t* blk = rblk + s * kRb;
+      if (live) {
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int k = kh + c;
+          const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
+          *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, r)) = __float2bfloat16_rn(v);
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&rready[s]);
+    }
+    if (!ok) atomicExch(cta_err, 1);
   } else if (warp >= 2) {
-    // ---- forward (8 warps), residual (warp 2), run drain (warps 2-5) -------
+    // ---- forward (8 warps), run drain (all 8) -------------------------------
     const int fw = warp - 2;
     const int nks = (int)(a.ld / 128);          // 16-feature steps of this warp
     const int f0 = fw * nks * 16;               // first feature of this warp
@@ -250,20 +315,15 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         }
       }
     // ldmatrix row of this lane: matrix m = lane / 8 (rows 8 (m & 1) .., features 8 (m >> 1) ..)
-    const int lr = ((lane >> 3) & 1) * 8 + (lane & 7), lk = (lane >> 4) * 8;
-    // Every forward warp goes through every tile's named barrier, also after
-    // a failed wait (it then skips its waits and writes), so none is left
-    // waiting at the barrier.
+    // (8-row tiles: rows 8-15 of the fragment repeat rows 0-7 and are ignored)
+    const int lr = (((lane >> 3) & 1) * 8 + (lane & 7)) & (kRR - 1), lk = (lane >> 4) * 8;
     bool ok = true;
     int run = 0;
     for (int i = 0; i < n; ++i) {
       const int s = i % S;
       const int4 tl = a.tiles[t0 + i];
       const bool last = (tl.w & 2) || i == n - 1;
-      // the residual warp's label, fetched before the tile's work
-      int lab = -1;
-      if (warp == 2 && (lane >> 1) < tl.y) lab = a.y[tl.x + (lane >> 1)];
-      if (ok && !__all_sync(0xffffffffu, mbar_wait(&full[s], (i / S) & 1, a.status))) ok = false;
+      if (!__all_sync(0xffffffffu, mbar_wait(&full[s], (i / S) & 1, a.status))) { ok = false; break; }
       const uint32_t xs = smem_u32(sm + (size_t)s * L.slot_bytes);
       // four independent accumulator chains (class halves x even / odd steps)
       float c0[4] = {0.f, 0.f, 0.f, 0.f}, c1[4] = {0.f, 0.f, 0.f, 0.f};
@@ -272,7 +332,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       for (int ks = 0; ks < kMaxKs; ++ks) {
         if (ks < nks) {
           const int f = f0 + ks * 16 + lk;
-          const uint32_t ad = xs + (uint32_t)((f >> 6) * 2048 + lr * 128 + ((((f & 63) >> 3) ^ (lr & 7)) << 4));
+          const uint32_t ad = xs + (uint32_t)((f >> 6) * kBlk + lr * 128 + ((((f & 63) >> 3) ^ (lr & 7)) << 4));
           uint32_t a0, a1, a2, a3;
           ldsm_x4(ad, a0, a1, a2, a3);
           if (ks & 1) {
@@ -289,61 +349,19 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         c0[j] += d0[j];
         c1[j] += d1[j];
       }
-      // partial logits: rows g, g + 8; classes 2tq, 2tq + 1 (+ 8 for c1)
+      // partial logits: rows g (and g + 8 for 16-row tiles); classes 2tq, 2tq + 1 (+ 8 for c1)
       float* zp = zpart + (size_t)(s * kFw + fw) * (kRR * 16);
       *reinterpret_cast<float2*>(zp + g * 16 + 2 * tq) = make_float2(c0[0], c0[1]);
-      *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 2 * tq) = make_float2(c0[2], c0[3]);
       *reinterpret_cast<float2*>(zp + g * 16 + 8 + 2 * tq) = make_float2(c1[0], c1[1]);
-      *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 8 + 2 * tq) = make_float2(c1[2], c1[3]);
-      named_sync(1, 32 * kFw);
-      if (warp == 2) {
-        // lane: row lane / 2, classes 8 (lane & 1) .. + 7
-        const int r = lane >> 1, kh = (lane & 1) * 8;
-        float z[8];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) z[c] = 0.f;
-        const float* zs = zpart + (size_t)s * kFw * (kRR * 16) + r * 16 + kh;
-#pragma unroll
-        for (int w = 0; w < kFw; ++w) {
-          const float4 u0 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16));
-          const float4 u1 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16) + 4);
-          z[0] += u0.x; z[1] += u0.y; z[2] += u0.z; z[3] += u0.w;
-          z[4] += u1.x; z[5] += u1.y; z[6] += u1.z; z[7] += u1.w;
-        }
-        float m = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          if (kh + c < a.K) m = fmaxf(m, z[c]);
-        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-        float e[8], sum = 0.f;
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          e[c] = kh + c < a.K ? expf(z[c] - m) : 0.f;
-          sum += e[c];
-        }
-        sum += __shfl_xor_sync(0xffffffffu, sum, 1);
-        const bool valid = r < tl.y;
-        const float inv = 1.0f / sum;
-        // the MMAs of this slot's previous tile have read its R block
-        if (ok && i >= S && !__all_sync(0xffffffffu, mbar_wait(&empty[s], ((i / S) - 1) & 1, a.status))) ok = false;
-        if (ok) {
-          uint8_t* blk = rblk + s * kRb;
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const int k = kh + c;
-            const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
-            *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, r)) = __float2bfloat16_rn(v);
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&rready[s]);
-        }
+      if (kRR == 16) {
+        *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 2 * tq) = make_float2(c0[2], c0[3]);
+        *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 8 + 2 * tq) = make_float2(c1[2], c1[3]);
       }
-      if (last && ok) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&zready[s]);
+      if (last) {
         // end of this CTA's run in a partition: G^T slices -> one partial
-        if (!__all_sync(0xffffffffu, mbar_wait(acc_full, run & 1, a.status))) ok = false;
-      }
-      if (last && ok) {
+        if (!__all_sync(0xffffffffu, mbar_wait(acc_full, run & 1, a.status))) { ok = false; break; }
         // warps w and w + 4 share TMEM lane quarter w % 4 and split the
         // slices: pairs (2j, 2j + 1) go to the first, then the second, ...
         tc_fence_after();
