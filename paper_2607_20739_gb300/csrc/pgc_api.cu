@@ -128,8 +128,8 @@ struct pgc_ctx {
   bool tc = false;           // softmax on the tensor cores (bf16 features)
   bool smallk = false;       // few-class softmax: one-pass cluster kernel
   int sk_nper = 0;           // its 64-feature blocks per CTA slice
-  int sk_nc = 0;             // its clusters (whole-row variant: its CTAs)
-  bool sk_rows = false;      // the whole-row variant (one CTA per SM, kRowsTileRows-row tiles)
+  int sk_nc = 0;             // its clusters (whole-row variant: its CTAs, two per pair)
+  bool sk_rows = false;      // the whole-row variant (CTA pairs, kRowsTileRows-row tiles)
   int sk_slots = 0;          // its tile slots
   int sk_box = 1;            // its 64-feature blocks per TMA copy
   bool sk_tail = true;       // its fused commit + decode (PGC_NO_ROWS_TAIL=1: separate kernels)
@@ -269,7 +269,8 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
         ph.sk_tiles.push_back(0);
         te.push_back(e);
       }
-    const int64_t T = (int64_t)te.size(), nc = ctx->sk_nc;
+    // runs per cluster (whole-row variant: per CTA pair)
+    const int64_t T = (int64_t)te.size(), nc = ctx->sk_rows ? ctx->sk_nc / 2 : ctx->sk_nc;
     std::vector<int32_t> items_of(nE, 0);
     int item = 0;
     for (int64_t cl = 0; cl < nc; ++cl) {
@@ -486,19 +487,15 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     const char* env2 = std::getenv("PGC_NO_SMALLK");
     const char* env4 = std::getenv("PGC_NO_ROWS");
     if (!ctx->tc && dtype == PGC_BF16 && !(env2 && env2[0] == '1') && !(env4 && env4[0] == '1') && K <= 16) {
-      // few classes, rows short enough to hold 16 whole rows per slot: one
-      // CTA per SM, no exchange between CTAs (PGC_NO_ROWS=1 keeps the
-      // cluster kernel)
-      const int64_t ldr = (int64_t)align_up((size_t)d, 128);
+      // few classes, rows short enough to hold 16 whole rows per CTA pair
+      // and slot: one CTA per SM, a cluster of two per tile (PGC_NO_ROWS=1
+      // keeps the 8-CTA cluster kernel)
+      const int64_t ldr = (int64_t)align_up((size_t)d, 256);
       const int slots = rows_slots(ldr);
-      // TMA copies of up to 8 blocks (16 KB); PGC_ROWS_BOX sets the blocks per copy
-      int box = 1;
-      for (int b = 8; b >= 1; --b)
-        if ((ldr / 64) % b == 0) { box = b; break; }
-      if (const char* env = std::getenv("PGC_ROWS_BOX")) {
-        const int b = std::atoi(env);
-        if (b >= 1 && (ldr / 64) % b == 0) box = b;
-      }
+      // TMA copies of up to 8 blocks (16 KB); PGC_ROWS_BOX requests another count
+      int req = 0;
+      if (const char* env = std::getenv("PGC_ROWS_BOX")) req = std::atoi(env);
+      const int box = rows_box_blocks(ldr, req);
       ctx->sk_box = box;
       if (const char* env = std::getenv("PGC_NO_ROWS_TAIL")) ctx->sk_tail = env[0] != '1';
       // the occupancy query first: it makes the runtime's context current,

@@ -266,16 +266,15 @@ int smallk_max_clusters(int nper);
 cudaError_t launch_softmax_smallk(const void* tmX, const void* tmW, const SmallKArgs& a, int nclusters,
                                   cudaStream_t st);
 
-// ---- softmax with few classes, whole rows per CTA (softmax_rows.cu) --------
+// ---- softmax with few classes, whole rows per CTA pair (softmax_rows.cu) ---
 // tiles[i] = {first global X row, rows (<= kRowsTileRows), item, flags: 1 first / 2 last
-// tile of a CTA's run in one partition}; CTA c of G takes tiles
-// [ntiles c / G, ntiles (c + 1) / G).  partials[item][K][ld] receives the
-// unscaled gradient sums of the run.
+// tile of a pair's run in one partition}; pair p of Np (clusters of two CTAs,
+// one per half of the features) takes tiles [ntiles p / Np, ntiles (p + 1) / Np).
+// partials[item][K][ld] receives the unscaled gradient sums of the run.
 constexpr int kRowsTileRows = 16;
 constexpr int64_t kRowsMaxLd = 3072;       // the forward keeps a warp's W^T slice in registers
 constexpr int kRowsMaxSlots = 8;
-constexpr int kRowsTmemCols = 512;         // G^T: ld / 128 slices of 16 columns
-constexpr uint32_t kRowsSmemBudget = 227 * 1024 - 9 * 1024;   // the decode plan is static shared memory
+constexpr uint32_t kRowsSmemBudget = 227 * 1024 - 1024;   // a little static shared memory beside it
 struct RowsArgs {
   const int4* tiles;
   int ntiles;
@@ -284,7 +283,7 @@ struct RowsArgs {
   const uint16_t* wb;       // bf16 W [16][ld], zero rows past K
   float* partials;
   int64_t P;                // K * ld
-  int64_t ld;               // a multiple of 128, at most kRowsMaxLd
+  int64_t ld;               // a multiple of 256, at most kRowsMaxLd
   int nslots;
   int box_blocks;           // 64-feature blocks per TMA copy (divides ld / 64)
   int* status;
@@ -305,9 +304,12 @@ struct RowsArgs {
   int* counters = nullptr;
   DecodeArgs dec;
 };
-// Slots of kRowsTileRows x ld that fit (0: ld not supported).
+// Slots of kRowsTileRows x ld/2 (a CTA's half tile) that fit (0: ld not supported).
 int rows_slots(int64_t ld);
-// CTAs of the grid (one per SM; 0: cannot launch).
+// 64-feature blocks per TMA copy: `requested` if it divides a half tile's
+// blocks, else the largest such count up to 8.
+int rows_box_blocks(int64_t ld, int requested);
+// CTAs of the grid: two per co-resident cluster, one per SM (0: cannot launch).
 int rows_max_ctas(int64_t ld, int nslots);
 // tmX: X as [ld/64][rows][64] bf16 blocks, box {64, kRowsTileRows, box_blocks} (make_tmap_bf16_rows)
 cudaError_t launch_softmax_rows(const void* tmX, const RowsArgs& a, int nctas, cudaStream_t st);

@@ -1,32 +1,33 @@
 // Softmax gradient for few classes (K <= 16, §III with f = log sum_k
-// exp(w_k.x) - w_y.x), bf16 features, one pass over X, whole rows per CTA.
+// exp(w_k.x) - w_y.x), bf16 features, one pass over X, whole rows per CTA pair.
 //
 // For K this small both contractions of the gradient are thin:
 //   Z = X_tile W^T           (16 rows x 16 classes, summed over d)
 //   G += X_tile^T R          (d features x 16 classes, summed over the rows)
-// and the step is bound by reading X once.  Each CTA (one per SM) streams
-// tiles of kRR whole rows (kRR x ld bf16, laid out as 64-feature blocks of kRR
-// rows with 128-byte swizzle by 3-D TMA copies of box_blocks blocks each)
-// through a ring of slots; 8-row tiles keep four 48 KB slots in flight at
-// d = 3072 (the MMA shapes stay at 16 rows: the extra rows repeat the tile's
-// and carry zero residuals):
-//   1. eight warps form the logits with warp-level mma.sync (m16n8k16, bf16
-//      in, fp32 out), each over its d/8 features, with its slice of W^T held
-//      in registers for the whole step; the eight partial 16 x 16 blocks are
-//      summed through shared memory;
-//   2. a warp of its own forms R = softmax(Z) - onehot(y) (zero past K and
-//      past the partition's rows) in bf16, in the no-swizzle K-major operand
-//      layout, while the eight go on with the next tile;
+// and the step is bound by reading X once.  A cluster of two CTAs (one per
+// SM) streams 16-row tiles; CTA r holds the tile's features
+// [r ld/2, (r + 1) ld/2) (16 x ld/2 bf16, laid out as 64-feature blocks of 16
+// rows with 128-byte swizzle by 3-D TMA copies of box_blocks blocks each) in a
+// ring of slots, so four 48 KB slots are in flight at d = 3072:
+//   1. eight warps form the partial logits of the CTA's features with
+//      warp-level mma.sync (m16n8k16, bf16 in, fp32 out), each over a
+//      sixteenth of d, with its slice of W^T held in registers for the whole
+//      step, and hand them over through shared memory;
+//   2. a warp of its own sums them, sends the CTA's 16 x 16 block to the other
+//      CTA with st.async into distributed shared memory, adds the two blocks in
+//      rank order (so both CTAs form the same R) and forms R = softmax(Z) -
+//      onehot(y) (zero past K and past the partition's rows) in bf16, in the
+//      no-swizzle K-major operand layout;
 //   3. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
-//      the 16 rows; A = the resident X tile read MN-major) into a TMEM
-//      accumulator of G^T that spans the CTA's run of tiles in a partition,
-//      and frees the slot with tcgen05.commit.
-// No data leaves the CTA before the end of a run; then four warps write the
-// run's G^T as one partial (one item per CTA and partition).  With the fused
-// tail the same grid then commits (after a grid barrier: every CTA sums a
-// share of the partitions' items in item order, scales by 1/m_e and writes
-// the stores) and decodes (after a second barrier: coefficients from the
-// mask, decode and SGD over a share of the columns); otherwise separate
+//      the 16 rows; A = the resident half tile read MN-major) into a TMEM
+//      accumulator of the CTA's half of G^T that spans the pair's run of tiles
+//      in a partition, and frees the slot with tcgen05.commit.
+// No data leaves the pair before the end of a run; then the eight warps write
+// the run's G^T halves into one partial (one item per pair and partition).
+// With the fused tail the same grid then commits (after a grid barrier: every
+// CTA sums a share of the partitions' items in item order, scales by 1/m_e and
+// writes the stores) and decodes (after a second barrier: coefficients from
+// the mask, decode and SGD over a share of the columns); otherwise separate
 // commit and decode kernels follow.
 // Every wait is bounded; the TMEM allocation is released on every path.
 #include <cuda.h>
@@ -41,14 +42,18 @@ namespace pgc {
 namespace {
 
 constexpr int kRR = kRowsTileRows;       // rows per tile
-static_assert(kRR == 8 || kRR == 16, "tiles of 8 or 16 rows (mma.sync M = 16, tcgen05 K = 16)");
+static_assert(kRR == 16, "16-row tiles (mma.sync M = 16, tcgen05 K = 16)");
 constexpr uint32_t kBlk = kRR * 128;      // one 64-feature block of the tile
+constexpr int kPairCtas = 2;             // CTAs per cluster: feature halves
 constexpr int kFw = 8;                   // forward warps (warps 2..9)
-constexpr int kRWarp = 2 + kFw;          // the residual warp
-constexpr int kRThreads = 64 + 32 * kFw + 32;
-constexpr int kMaxKs = kRowsMaxLd / 128; // 16-feature steps per forward warp at the largest ld
-constexpr uint32_t kZp = kRR * 16 * 4;   // one warp's partial logits (kRR rows x 16 classes fp32)
-constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16; rows past kRR stay zero)
+constexpr int kRWarp = 2 + kFw;          // the residual warps (even and odd tiles)
+constexpr int kNRes = 2;
+constexpr int kRThreads = 64 + 32 * kFw + 32 * kNRes;
+// 16-feature steps per forward warp at the largest ld
+constexpr int kMaxKs = (int)(kRowsMaxLd / kPairCtas / (16 * kFw));
+constexpr uint32_t kZp = kRR * 16 * 4;   // a 16 x 16 fp32 block of partial logits
+constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16)
+constexpr int kTmemCols = 256;           // G^T half: ld / 256 slices of 16 columns
 
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
   uint64_t d = 0;
@@ -77,6 +82,43 @@ __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+// shared::cta address -> the same offset in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t mapa_u32(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_async_v4(uint32_t raddr, float4 v, uint32_t rbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   raddr),
+               "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t rbar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(rbar) : "memory");
+}
+__device__ __forceinline__ bool try_wait_cluster(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// bounded wait with cluster-scope acquire (the data came from the other CTA)
+__device__ __forceinline__ bool wait_cluster(uint64_t* bar, uint32_t parity, int* status) {
+  if (try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 0; it < kWaitMaxIters; ++it) {
+    if (try_wait_cluster(bar, parity)) return true;
+    if ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitMaxNs) break;
+  }
+  atomicOr(status, kErrWaitTimeout);
+  return false;
 }
 // Element (class k, tile row r) of the R block in the K-major layout without
 // swizzle: 8 x 8 core matrices (8 classes x 16 bytes of rows), the core of
@@ -117,44 +159,57 @@ __device__ bool grid_barrier(int* ctr, int* status, int* flag) {
 
 }  // namespace
 
+// Shared memory of a CTA: slots of its half tile, two sets (tile parity) of
+// the forward warps' partial logits (the fused tail's decode plan reuses
+// them), two blocks for the other CTA's partial, R blocks, barriers.
 struct RowsSmem {
-  uint32_t slot_bytes, zpart, rblk, bars, total;
+  uint32_t slot_bytes, zpart, zpeer, rblk, bars, total;
 };
+constexpr int kRowsBars = 3 * kRowsMaxSlots + 8 + 4;
 __host__ __device__ static RowsSmem rows_smem(int64_t ld, int nslots) {
   RowsSmem s;
-  s.slot_bytes = (uint32_t)(kRR * ld * 2);
+  s.slot_bytes = (uint32_t)(kRR * (ld / kPairCtas) * 2);
   s.zpart = (uint32_t)nslots * s.slot_bytes;
-  s.rblk = s.zpart + (uint32_t)nslots * kFw * kZp;
+  s.zpeer = s.zpart + 2 * kFw * kZp;
+  s.rblk = s.zpeer + 2 * kZp;
   s.bars = s.rblk + (uint32_t)nslots * kRb;
-  s.total = s.bars + (4 * kRowsMaxSlots + 4) * 8 + 16;
+  s.total = s.bars + kRowsBars * 8 + 16;
   return s;
 }
+static_assert(2 * kFw * kZp >= sizeof(DecodePlan), "the decode plan fits the partial-logit area");
 
 __global__ void __launch_bounds__(kRThreads, 1)
 softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ RowsArgs a) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ DecodePlan plan;
   __shared__ int bar_flag;
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = a.nslots;
   const RowsSmem L = rows_smem(a.ld, S);
-  float* zpart = reinterpret_cast<float*>(sm + L.zpart);
+  float* zpart = reinterpret_cast<float*>(sm + L.zpart);   // [2][kFw][16][16]
+  float* zpeer = reinterpret_cast<float*>(sm + L.zpeer);   // [2][16][16] from the other CTA
+  DecodePlan& plan = *reinterpret_cast<DecodePlan*>(zpart);  // the tail's, after the tiles
   uint8_t* rblk = sm + L.rblk;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.bars);
-  uint64_t* full = bars;                       // [S] X tile landed
-  uint64_t* empty = bars + kRowsMaxSlots;      // [S] the tile's MMAs are done (slot, R block free)
-  uint64_t* rready = bars + 2 * kRowsMaxSlots; // [S] R block written
-  uint64_t* zready = bars + 3 * kRowsMaxSlots; // [S] every forward warp's partial logits written
-  uint64_t* acc_full = bars + 4 * kRowsMaxSlots;
+  uint64_t* full = bars;                          // [S] half tile landed
+  uint64_t* empty = bars + kRowsMaxSlots;         // [S] the tile's MMAs are done (slot, R block free)
+  uint64_t* rready = bars + 2 * kRowsMaxSlots;    // [S] R block written
+  uint64_t* zready = bars + 3 * kRowsMaxSlots;    // [2] every forward warp's partial written
+  uint64_t* zfree = zready + 2;                   // [2] the residual warp has read them
+  uint64_t* zpeer_full = zready + 4;              // [2] the other CTA's block arrived
+  uint64_t* zpeer_empty = zready + 6;             // [2] the other CTA has read this CTA's block
+  uint64_t* acc_full = zready + 8;
   uint64_t* acc_empty = acc_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 2);
   int* cta_err = reinterpret_cast<int*>(acc_full + 3);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nmt = (int)(a.ld / 128);           // 128-feature M slices of the backward
-  // this CTA's tiles: [T c / G, T (c + 1) / G)
-  const int t0 = (int)((int64_t)a.ntiles * blockIdx.x / gridDim.x);
-  const int t1 = (int)((int64_t)a.ntiles * (blockIdx.x + 1) / gridDim.x);
+  const int rank = (int)cluster_rank();
+  const int64_t ldh = a.ld / kPairCtas;          // features of this CTA
+  const int nmt = (int)(ldh / 128);              // 128-feature M slices of the backward
+  // this pair's tiles: [T p / Np, T (p + 1) / Np)
+  const int pair = (int)blockIdx.x / kPairCtas, npairs = (int)gridDim.x / kPairCtas;
+  const int t0 = (int)((int64_t)a.ntiles * pair / npairs);
+  const int t1 = (int)((int64_t)a.ntiles * (pair + 1) / npairs);
   const int n = t1 - t0;
 
   if (threadIdx.x == 0) {
@@ -163,34 +218,39 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
       mbar_init(&rready[s], 1);
-      mbar_init(&zready[s], kFw);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&zready[b], kFw);
+      mbar_init(&zfree[b], 1);
+      mbar_init(&zpeer_full[b], 1);
+      mbar_init(&zpeer_empty[b], 1);
     }
     mbar_init(acc_full, 1);
     mbar_init(acc_empty, kFw);
     fence_mbar_init();
   }
-  // R blocks start zeroed: with 8-row tiles their rows 8-15 stay zero
-  for (uint32_t k = threadIdx.x; k < (uint32_t)S * kRb / 16; k += blockDim.x)
-    reinterpret_cast<uint4*>(rblk)[k] = make_uint4(0u, 0u, 0u, 0u);
-  fence_proxy_async_smem();
   if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                 "r"((uint32_t)kRowsTmemCols)
+                 "r"((uint32_t)kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  tc_fence_before();
   __syncthreads();
+  // the other CTA's first two blocks may arrive before this CTA reaches them
+  if (threadIdx.x == 0)
+    for (int b = 0; b < 2 && b < n; ++b) mbar_arrive_expect_tx(&zpeer_full[b], kZp);
+  tc_fence_before();
+  cluster_sync_all();                    // both CTAs' barriers exist before any st.async
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   if (threadIdx.x == 0) grid_dep_launch();
 
   if (warp == 0 && lane == 0) {
-    // ---- producer: one 3-D copy per tile ------------------------------------
+    // ---- producer: this CTA's half of each tile ------------------------------
     bool ok = true;
     int issued = 0;
     const uint32_t bytes = L.slot_bytes;
-    const int nkb = (int)(a.ld / 64);
+    const int nkb = (int)(ldh / 64), kb0 = rank * nkb;
     // X does not change between steps: no wait for the previous kernel
     for (int i = 0; i < n && ok; ++i) {
       const int s = i % S;
@@ -198,7 +258,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       mbar_arrive_expect_tx(&full[s], bytes);
       const int row0 = a.tiles[t0 + i].x;
       for (int z = 0; z < nkb; z += a.box_blocks)
-        tma_load_3d(sm + (size_t)s * bytes + (size_t)z * kBlk, &tmX, 0, row0, z, &full[s]);
+        tma_load_3d(sm + (size_t)s * bytes + (size_t)z * kBlk, &tmX, 0, row0, kb0 + z, &full[s]);
       ++issued;
     }
     if (!ok) atomicExch(cta_err, 1);
@@ -207,7 +267,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       mbar_wait(&full[s], (last / S) & 1, a.status);
     }
   } else if (warp == 1 && lane == 0) {
-    // ---- backward MMAs: G^T[f][k] += sum_r X[r][f] R[r][k] ----------------------
+    // ---- backward MMAs: G^T[f][k] += sum_r X[r][f] R[r][k] ------------------
     constexpr uint32_t id_bwd = idesc_bf16_f32(128, 16, true, false);
     bool ok = true;
     int run = 0;
@@ -223,11 +283,10 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       tc_fence_after();
       const uint32_t xs = smem_u32(sm + (size_t)s * L.slot_bytes);
       const uint64_t db = sdesc(smem_u32(rblk + s * kRb), 256, 128, 0);
-      // slice mt: two 64-feature blocks kBlk apart; the K = 16 rows of one
-      // MMA are two 8-row groups 1 KB apart (16-row tiles) or the tile's 8
-      // rows twice (8-row tiles: R's rows 8-15 are zero); slices 2 kBlk
-      // apart (the address field counts 16-byte units)
-      const uint64_t da0 = sdesc(xs, kBlk, kRR == 16 ? 1024 : 0, 2);
+      // slice mt: two 64-feature blocks kBlk apart, the K = 16 rows two 8-row
+      // groups 1 KB apart; slices 2 kBlk apart (the address field counts
+      // 16-byte units)
+      const uint64_t da0 = sdesc(xs, kBlk, 1024, 2);
       constexpr uint64_t kStep = (2 * kBlk) >> 4;
       if (first) {
         for (int mt = 0; mt < nmt; ++mt) umma_bf16_fresh(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)mt * kStep, db, id_bwd);
@@ -241,24 +300,27 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       }
     }
     if (!ok) atomicExch(cta_err, 1);
-  } else if (warp == kRWarp) {
-    // ---- residual: R = softmax(Z) - onehot(y) per tile --------------------
-    // lane: row lane / 2 (rows past kRR: idle lanes), classes 8 (lane & 1) .. + 7.
-    // zpart[s] and the R block of slot s are free again once the tile's slot
-    // was refilled (its full wait implies the previous MMAs completed).
-    const int r = (lane >> 1) & (kRR - 1), kh = (lane & 1) * 8;
-    const bool live = (lane >> 1) < kRR;
+  } else if (warp >= kRWarp) {
+    // ---- residual: the pair's logits, R = softmax(Z) - onehot(y) ------------
+    // Two warps, for the even and the odd tiles (every buffer and barrier of
+    // the exchange is per tile parity), so one tile's exchange with the other
+    // CTA overlaps the next tile's.  lane: row lane / 2, classes 8 (lane & 1)
+    // .. + 7.  The R block of slot s is free again once the tile's half was
+    // loaded (its full wait, through the forward warps' zready, implies the
+    // slot's previous MMAs completed).
+    const int r = lane >> 1, kh = (lane & 1) * 8;
+    const uint32_t peer = (uint32_t)(rank ^ 1);
     bool ok = true;
-    for (int i = 0; i < n && ok; ++i) {
-      const int s = i % S;
+    for (int i = warp - kRWarp; i < n && ok; i += kNRes) {
+      const int s = i % S, b = i & 1;
       const int4 tl = a.tiles[t0 + i];
-      const bool valid = live && r < tl.y;
-      const int lab = valid ? a.y[tl.x + r] : -1;        // fetched before the wait
-      if (!__all_sync(0xffffffffu, mbar_wait(&zready[s], (i / S) & 1, a.status))) { ok = false; break; }
+      const bool valid = r < tl.y;
+      const int lab = valid ? a.y[tl.x + r] : -1;        // fetched before the waits
+      if (!__all_sync(0xffffffffu, mbar_wait(&zready[b], (i >> 1) & 1, a.status))) { ok = false; break; }
       float z[8];
 #pragma unroll
       for (int c = 0; c < 8; ++c) z[c] = 0.f;
-      const float* zs = zpart + (size_t)s * kFw * (kRR * 16) + r * 16 + kh;
+      const float* zs = zpart + (size_t)b * kFw * (kRR * 16) + r * 16 + kh;
 #pragma unroll
       for (int w = 0; w < kFw; ++w) {
         const float4 u0 = *reinterpret_cast<const float4*>(zs + w * (kRR * 16));
@@ -266,6 +328,37 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         z[0] += u0.x; z[1] += u0.y; z[2] += u0.z; z[3] += u0.w;
         z[4] += u1.x; z[5] += u1.y; z[6] += u1.z; z[7] += u1.w;
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&zfree[b]);             // the forward warps may refill zpart[b]
+      // this CTA's block to the other CTA, once it has read the one sent two tiles ago
+      if (i >= 2 && !__all_sync(0xffffffffu, wait_cluster(&zpeer_empty[b], ((i >> 1) - 1) & 1, a.status))) {
+        ok = false;
+        break;
+      }
+      {
+        const uint32_t dst = mapa_u32(smem_u32(zpeer + (size_t)b * (kRR * 16) + r * 16 + kh), peer);
+        const uint32_t rbar = mapa_u32(smem_u32(&zpeer_full[b]), peer);
+        st_async_v4(dst, make_float4(z[0], z[1], z[2], z[3]), rbar);
+        st_async_v4(dst + 16, make_float4(z[4], z[5], z[6], z[7]), rbar);
+      }
+      if (!__all_sync(0xffffffffu, wait_cluster(&zpeer_full[b], (i >> 1) & 1, a.status))) { ok = false; break; }
+      const float* zp = zpeer + (size_t)b * (kRR * 16) + r * 16 + kh;
+      float y[8];
+      {
+        const float4 u0 = *reinterpret_cast<const float4*>(zp);
+        const float4 u1 = *reinterpret_cast<const float4*>(zp + 4);
+        y[0] = u0.x; y[1] = u0.y; y[2] = u0.z; y[3] = u0.w; y[4] = u1.x; y[5] = u1.y; y[6] = u1.z; y[7] = u1.w;
+      }
+      __syncwarp();
+      if (i + 2 < n) {
+        if (lane == 0) {
+          mbar_arrive_expect_tx(&zpeer_full[b], kZp);     // the other CTA's block of tile i + 2
+          mbar_arrive_remote(mapa_u32(smem_u32(&zpeer_empty[b]), peer));
+        }
+      }
+      // the same sum in both CTAs: rank 0's block first
+#pragma unroll
+      for (int c = 0; c < 8; ++c) z[c] = rank == 0 ? z[c] + y[c] : y[c] + z[c];
       float m = -INFINITY;
 #pragma unroll
       for (int c = 0; c < 8; ++c)
@@ -280,13 +373,11 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       sum += __shfl_xor_sync(0xffffffffu, sum, 1);
       const float inv = 1.0f / sum;
       uint8_t* blk = rblk + s * kRb;
-      if (live) {
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int k = kh + c;
-          const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
-          *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, r)) = __float2bfloat16_rn(v);
-        }
+      for (int c = 0; c < 8; ++c) {
+        const int k = kh + c;
+        const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
+        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, r)) = __float2bfloat16_rn(v);
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -294,10 +385,10 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     }
     if (!ok) atomicExch(cta_err, 1);
   } else if (warp >= 2) {
-    // ---- forward (8 warps), run drain (all 8) -------------------------------
+    // ---- forward (8 warps), run drain (all 8) ---------------------------------
     const int fw = warp - 2;
-    const int nks = (int)(a.ld / 128);          // 16-feature steps of this warp
-    const int f0 = fw * nks * 16;               // first feature of this warp
+    const int nks = (int)(ldh / (16 * kFw));    // 16-feature steps of this warp
+    const int f0 = fw * nks * 16;               // first feature of this warp within the half
     const int g = lane >> 2, tq = lane & 3;
     grid_dep_wait();                            // W is the previous step's update
     // B fragments of W^T for this warp's features: b0 = W[n][k0 + 2tq ..],
@@ -309,18 +400,17 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       for (int nb = 0; nb < 2; ++nb) {
         wf[ks][nb][0] = wf[ks][nb][1] = 0u;
         if (ks < nks) {
-          const uint16_t* wr = a.wb + (int64_t)(8 * nb + g) * a.ld + f0 + ks * 16 + 2 * tq;
+          const uint16_t* wr = a.wb + (int64_t)(8 * nb + g) * a.ld + rank * ldh + f0 + ks * 16 + 2 * tq;
           wf[ks][nb][0] = *reinterpret_cast<const uint32_t*>(wr);
           wf[ks][nb][1] = *reinterpret_cast<const uint32_t*>(wr + 8);
         }
       }
     // ldmatrix row of this lane: matrix m = lane / 8 (rows 8 (m & 1) .., features 8 (m >> 1) ..)
-    // (8-row tiles: rows 8-15 of the fragment repeat rows 0-7 and are ignored)
-    const int lr = (((lane >> 3) & 1) * 8 + (lane & 7)) & (kRR - 1), lk = (lane >> 4) * 8;
+    const int lr = ((lane >> 3) & 1) * 8 + (lane & 7), lk = (lane >> 4) * 8;
     bool ok = true;
     int run = 0;
     for (int i = 0; i < n; ++i) {
-      const int s = i % S;
+      const int s = i % S, b = i & 1;
       const int4 tl = a.tiles[t0 + i];
       const bool last = (tl.w & 2) || i == n - 1;
       if (!__all_sync(0xffffffffu, mbar_wait(&full[s], (i / S) & 1, a.status))) { ok = false; break; }
@@ -349,24 +439,28 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         c0[j] += d0[j];
         c1[j] += d1[j];
       }
-      // partial logits: rows g (and g + 8 for 16-row tiles); classes 2tq, 2tq + 1 (+ 8 for c1)
-      float* zp = zpart + (size_t)(s * kFw + fw) * (kRR * 16);
+      // the residual warp has read this buffer's previous tile (i - 2)
+      if (i >= 2 && !__all_sync(0xffffffffu, mbar_wait(&zfree[b], ((i >> 1) - 1) & 1, a.status))) {
+        ok = false;
+        break;
+      }
+      // partial logits: rows g, g + 8; classes 2tq, 2tq + 1 (+ 8 for c1)
+      float* zp = zpart + (size_t)(b * kFw + fw) * (kRR * 16);
       *reinterpret_cast<float2*>(zp + g * 16 + 2 * tq) = make_float2(c0[0], c0[1]);
       *reinterpret_cast<float2*>(zp + g * 16 + 8 + 2 * tq) = make_float2(c1[0], c1[1]);
-      if (kRR == 16) {
-        *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 2 * tq) = make_float2(c0[2], c0[3]);
-        *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 8 + 2 * tq) = make_float2(c1[2], c1[3]);
-      }
+      *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 2 * tq) = make_float2(c0[2], c0[3]);
+      *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 8 + 2 * tq) = make_float2(c1[2], c1[3]);
       __syncwarp();
-      if (lane == 0) mbar_arrive(&zready[s]);
+      if (lane == 0) mbar_arrive(&zready[b]);
       if (last) {
-        // end of this CTA's run in a partition: G^T slices -> one partial
+        // end of the pair's run in a partition: this CTA's G^T slices -> its
+        // half of the run's partial
         if (!__all_sync(0xffffffffu, mbar_wait(acc_full, run & 1, a.status))) { ok = false; break; }
         // warps w and w + 4 share TMEM lane quarter w % 4 and split the
         // slices: pairs (2j, 2j + 1) go to the first, then the second, ...
         tc_fence_after();
         const int q = warp & 3, half = (warp - 2) >> 2;
-        float* dst = a.partials + (int64_t)tl.z * a.P;
+        float* dst = a.partials + (int64_t)tl.z * a.P + rank * ldh;
         for (int mt = 2 * half; mt < nmt; mt += 4) {
           uint32_t gv[32];
           tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * 16), gv);   // slices mt, mt + 1
@@ -390,6 +484,9 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     if (!ok) atomicExch(cta_err, 1);
   }
   __syncthreads();
+  tc_fence_before();
+  cluster_sync_all();                    // no st.async or remote arrive is still aimed at this CTA
+  tc_fence_after();
   if (a.tail && !*cta_err) {
     // ---- fused tail: commit, then decode + SGD --------------------------------
     if (warp == 0) derive_plan_warp(a.dec, plan, lane);   // needs only the mask
@@ -440,7 +537,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     }
     __syncwarp();
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kRowsTmemCols)
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kTmemCols)
                  : "memory");
   }
 }
@@ -449,44 +546,63 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
 // host side
 // ---------------------------------------------------------------------------
 int rows_slots(int64_t ld) {
-  if (ld % 128 != 0 || ld > kRowsMaxLd) return 0;
+  if (ld % (128 * kPairCtas) != 0 || ld > kRowsMaxLd) return 0;
   int s = kRowsMaxSlots;
   while (s >= 2 && rows_smem(ld, s).total + 1024 > kRowsSmemBudget) --s;
   return s >= 2 ? s : 0;
 }
 
+int rows_box_blocks(int64_t ld, int requested) {
+  const int nkb = (int)(ld / kPairCtas / 64);   // blocks of one CTA's half
+  if (nkb < 1) return 0;
+  if (requested >= 1 && nkb % requested == 0) return requested;
+  for (int b = 8; b >= 1; --b)
+    if (nkb % b == 0) return b;
+  return 1;
+}
+
 static size_t rows_smem_bytes(int64_t ld, int nslots) { return 1024 + rows_smem(ld, nslots).total; }
+
+static cudaLaunchConfig_t rows_config(int64_t ld, int nslots, int nctas, cudaLaunchAttribute* attr, bool pdl,
+                                      cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)nctas);
+  cfg.blockDim = dim3(kRThreads);
+  cfg.dynamicSmemBytes = rows_smem_bytes(ld, nslots);
+  cfg.stream = st;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kPairCtas;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 2 : 1;
+  return cfg;
+}
 
 int rows_max_ctas(int64_t ld, int nslots) {
   const size_t smem = rows_smem_bytes(ld, nslots);
   if (cudaFuncSetAttribute(softmax_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
       cudaSuccess)
     return 0;
-  int per_sm = 0, sms = 0, dev = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, softmax_rows_kernel, kRThreads, smem) != cudaSuccess)
-    return 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
-                                                cudaSuccess)
-    return 0;
-  return per_sm >= 1 ? sms : 0;   // one CTA per SM (tensor memory)
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = rows_config(ld, nslots, kPairCtas, attr, false, 0);
+  int nc = 0;
+  if (cudaOccupancyMaxActiveClusters(&nc, softmax_rows_kernel, &cfg) != cudaSuccess) return 0;
+  return nc * kPairCtas;   // every pair co-resident (the fused tail's grid barriers need it)
 }
 
 cudaError_t launch_softmax_rows(const void* tmX, const RowsArgs& a, int nctas, cudaStream_t st) {
   if (a.ntiles <= 0) return cudaSuccess;
-  if (nctas < 1 || a.nslots < 2 || a.nslots > kRowsMaxSlots) return cudaErrorInvalidValue;
+  if (nctas < kPairCtas || nctas % kPairCtas != 0 || a.nslots < 2 || a.nslots > kRowsMaxSlots)
+    return cudaErrorInvalidValue;
+  if (a.box_blocks < 1 || (a.ld / kPairCtas / 64) % a.box_blocks != 0) return cudaErrorInvalidValue;
   const size_t smem = rows_smem_bytes(a.ld, a.nslots);
   cudaError_t e = cudaFuncSetAttribute(softmax_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)nctas);
-  cfg.blockDim = dim3(kRThreads);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = a.pdl ? 1 : 0;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = rows_config(a.ld, a.nslots, nctas, attr, a.pdl != 0, st);
   CUtensorMap x;
   std::memcpy(&x, tmX, sizeof(CUtensorMap));
   return cudaLaunchKernelEx(&cfg, softmax_rows_kernel, x, a);
