@@ -78,6 +78,34 @@ def test_parity_cluster_few_class_kernel(libpgc, cuda, monkeypatch, name):
     g.close()
 
 
+@pytest.mark.parametrize("run", ["1", "3", "8"])
+def test_parity_gradient_runs(libpgc, cuda, monkeypatch, run):
+    """The tensor-core gradient contraction with runs of 1, 3 and 8 partitions
+    per output tile (5 evaluated partitions: a shorter last run, or one run
+    holding them all); each run's sum goes into the slot total once."""
+    monkeypatch.setenv("PGC_GRAD_RUN", run)
+    w, T = WL["cr_n128_softmax_k1000"].replace(n=5, s=2, K=260, d=300, m=(70, 129, 1, 64, 200)), 5
+    Xs, ys, masks = generate(w, T)
+    g, grecs = run_gpu(libpgc, w, Xs, ys, masks)
+    assert g.gradient_path == "tc_fused"
+    orecs = run_oracle(w, Xs, ys, masks)
+    compare_runs(w, grecs, orecs)
+    g.close()
+
+
+def test_parity_unfused_tensor_core_path(libpgc, cuda, monkeypatch):
+    """A class count the fused kernel covers, forced through the three-kernel
+    fall-back (logits GEMM, residual kernel, gradient contraction)."""
+    monkeypatch.setenv("PGC_NO_FUSED", "1")
+    w, T = CASES["cr_tc_k300_d320_m200"]
+    Xs, ys, masks = generate(w, T)
+    g, grecs = run_gpu(libpgc, w, Xs, ys, masks)
+    assert g.gradient_path == "tc"
+    orecs = run_oracle(w, Xs, ys, masks)
+    compare_runs(w, grecs, orecs)
+    g.close()
+
+
 def test_stores_hold_the_scheduled_gradients(libpgc, cuda):
     """After each step every worker's store slot l holds the gradient of its
     slot-l partition at the step it was last evaluated (s(t,i,j), §V-B)."""
