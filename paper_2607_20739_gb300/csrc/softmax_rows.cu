@@ -13,11 +13,11 @@
 //      warp-level mma.sync (m16n8k16, bf16 in, fp32 out), each over a
 //      sixteenth of d, with its slice of W^T held in registers for the whole
 //      step, and hand them over through shared memory;
-//   2. a warp of its own sums them, sends the CTA's 16 x 16 block to the other
-//      CTA with st.async into distributed shared memory, adds the two blocks in
-//      rank order (so both CTAs form the same R) and forms R = softmax(Z) -
-//      onehot(y) (zero past K and past the partition's rows) in bf16, in the
-//      no-swizzle K-major operand layout;
+//   2. two warps of their own (even and odd tiles) sum them, send the CTA's
+//      16 x 16 block to the other CTA with st.async into distributed shared
+//      memory, add the two blocks in rank order (so both CTAs form the same
+//      R) and form R = softmax(Z) - onehot(y) (zero past K and past the
+//      partition's rows) in bf16, in the no-swizzle K-major operand layout;
 //   3. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
 //      the 16 rows; A = the resident half tile read MN-major) into a TMEM
 //      accumulator of the CTA's half of G^T that spans the pair's run of tiles

@@ -1,7 +1,8 @@
 // Logits GEMM with the softmax residual in its epilogue (§III with f = log
 // sum_k exp(w_k.x) - w_y.x): for every 128-row tile of the evaluated
 // partitions, R = softmax(X Wb^T) - onehot(y) in bf16, written straight to
-// the R buffer that the gradient GEMM reads; the logits never leave the chip.
+// the R buffer that the gradient contraction reads; the logits never leave
+// the chip.
 //
 // A cluster of NT CTAs (NT = padded classes / 256, one 256-class N tile each)
 // computes one row tile at a time.  The X tile is common to the cluster: each
@@ -17,9 +18,10 @@
 //   pass 2  r = exp(z - M) / S - [class == y] with the row's combined M, S,
 //   rounded to bf16, staged as 32 x 64 boxes in swizzled shared memory and
 //   written with TMA stores.  Rows past the partition and classes past K
-//   inside a box are written as zeros (the gradient GEMM reads whole 64-row
-//   blocks); boxes wholly past K are not written (the buffer starts zeroed).
-// The grid also zeroes the slot total that the gradient GEMM accumulates into.
+//   inside a box are written as zeros (the gradient contraction reads whole
+//   64-row blocks); boxes wholly past K are not written (the buffer starts
+//   zeroed).  The grid also zeroes the slot total that the gradient
+//   contraction accumulates into.
 // Every wait is bounded; the cluster barrier at the end keeps every CTA alive
 // until no peer can still write into it.
 #include <cuda.h>
@@ -337,11 +339,9 @@ tc_logits_softmax_kernel(const __grid_constant__ CUtensorMap tmXq, const __grid_
 static size_t fused_smem_bytes(int NT) { return 1024 + fused_smem(NT).total; }
 
 static cudaError_t fused_attributes(int NT) {
-  cudaError_t e = cudaFuncSetAttribute(tc_logits_softmax_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)fused_smem_bytes(NT));
-  if (e == cudaSuccess && NT > 8)
-    e = cudaFuncSetAttribute(tc_logits_softmax_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-  return e;
+  // clusters of at most 8 CTAs (kMaxNT): the portable size, no opt-in needed
+  return cudaFuncSetAttribute(tc_logits_softmax_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)fused_smem_bytes(NT));
 }
 
 int tc_softmax_max_clusters(int NT) {
