@@ -39,6 +39,22 @@ Baselines (§VI-A), for comparison on the same kernels: IS-SGD (the master
 averages the n - s fastest workers' own-partition gradients) and GC with FR
 placement (every worker evaluates its c partitions every step).
 
+§V-A, the naive pipelined construction on cyclic repetition: PGC-CR's
+schedule and placement, but each worker uploads GC-CR's weighted sum
+sum_l c_{j,l} * (its latest copy of g_{(j+l) mod n}) and the master applies
+GC-CR's straggler-dependent decode weights d_m(J); alpha_{m,k} = d_m c_{j_m,l}
+are the decoding coefficients whose range §V-A tracks.  The coefficients
+c_{j,l} are those of the cyclic-repetition construction of gradient coding,
+which §V-A cites (Tandon et al., ICML 2017) without restating; it is
+restated below from its definition.  With every copy current (GC-CR proper:
+all c partitions evaluated each step) the decode is exact.  Further readings:
+  R14 the naive and GC-CR decodes are scaled by 1/n, like FR's, so that with
+      current copies they equal DGD's (1/n) sum_k g_k;
+  R15 the construction's random matrix arrives as draws [s][n-1]; its last
+      column is minus the row sums (so H 1 = 0);
+  R16 the range of alpha is taken over the pairs the definition names:
+      received workers j_m and the c partitions each holds.
+
 Parity of whole trajectories is pinned only through the invariants the paper
 proves (eq. cr-fullsum, eq. cr-unbiased, the FR / GC equivalence and the DGD
 special case); there is no printed trajectory to compare with.
@@ -242,6 +258,63 @@ def appearance_counts(scheme: int, n: int, s: int, mask) -> np.ndarray:
 
 
 # ----------------------------------------------------------------------------
+# GC-CR encoding and decoding coefficients (§V-A)
+# ----------------------------------------------------------------------------
+
+def gc_cr_encoding(n: int, s: int, draws=None) -> np.ndarray:
+    """Encoding matrix B [n][n] of gradient coding with cyclic repetition.
+
+    The construction §V-A cites (Tandon et al. 2017, cyclic repetition):
+    H = [draws | -(row sums of draws)] is s x n, so H 1 = 0.  Row j of B is
+    supported on {j, j+1, ..., j+s} mod n, has B[j][j] = 1, and its other s
+    entries x solve H[:, {j+1..j+s}] x = -H[:, j]; then H B[j]^T = 0.  So the
+    rows of B and the all-ones vector all lie in the null space of H, which
+    has dimension n - s for generic draws, and any n - s rows of B span it:
+    the master can always find d with sum_m d_m B[j_m] = 1.
+    Worker j's encoding coefficient c_{j,l} is B[j][(j + l) mod n].
+    """
+    B = np.zeros((n, n), dtype=np.float64)
+    if s == 0:
+        np.fill_diagonal(B, 1.0)
+        return B
+    D = _as64(draws).reshape(s, n - 1)
+    H = np.concatenate([D, -D.sum(axis=1, keepdims=True)], axis=1)
+    for j in range(n):
+        rest = [(j + l) % n for l in range(1, s + 1)]
+        B[j, j] = 1.0
+        B[j, rest] = np.linalg.solve(H[:, rest], -H[:, j])
+    return B
+
+
+def encoding_coefficients(B: np.ndarray, c: int) -> np.ndarray:
+    """c_{j,l} = B[j][(j + l) mod n] for l = 0..c-1 (§V-A), shape [n][c]."""
+    n = B.shape[0]
+    return np.array([[B[j, (j + l) % n] for l in range(c)] for j in range(n)])
+
+
+def gc_decode_weights(B: np.ndarray, mask) -> np.ndarray:
+    """GC-CR's decode weights d(J) (§V-A): sum_{m} d_m B[j_m] = 1 over the
+    received workers J; d is 0 for stragglers.  Raises if no such d exists."""
+    n = B.shape[0]
+    J = received_set(mask)
+    A = B[J, :].T                                      # n equations, |J| unknowns
+    sol, _, rank, _ = np.linalg.lstsq(A, np.ones(n), rcond=None)
+    scale = 1.0 + np.abs(sol).max() * np.abs(A).max() if len(J) else 1.0
+    if rank < len(J) or np.abs(A @ sol - 1.0).max() > 1e-8 * scale:
+        raise ValueError("this encoding cannot decode the straggler pattern")
+    d = np.zeros(n)
+    d[J] = sol
+    return d
+
+
+def decoding_alpha(B: np.ndarray, d: np.ndarray, mask, c: int) -> dict:
+    """alpha_{m,k} = d_m c_{j_m,l} with (j_m + l) mod n = k (§V-A), keyed
+    (j_m, k), for every received worker j_m and each partition it holds."""
+    n = B.shape[0]
+    return {(j, (j + l) % n): d[j] * B[j, (j + l) % n] for j in received_set(mask) for l in range(c)}
+
+
+# ----------------------------------------------------------------------------
 # The PGC training loop, literally per worker (§IV-A, §V-B, §VI-A)
 # ----------------------------------------------------------------------------
 
@@ -419,12 +492,67 @@ class GCFROracle:
         return self.inner.loss_value()
 
 
-def run_mode(mode, scheme, n, s, loss, Xs, ys, lr, masks, beta0=None, K=1, record_loss=True):
-    """run() for a training mode: "pgc", "is_sgd" or "gc" (GC with FR placement)."""
+class NaiveCROracle(PGCOracle):
+    """The naive PGC-CR construction of §V-A (pipelined=True): PGC-CR's
+    rotation and stores, GC-CR's weighted uploads and decode weights.  With
+    pipelined=False every worker evaluates all c partitions every step: GC
+    with cyclic repetition, the exact scheme the naive one pipelines.
+
+    draws: the construction's random numbers, [s][n-1] (reading R15).
+    """
+
+    def __init__(self, n, s, loss, Xs, ys, lr, draws=None, beta0=None, K=1, pipelined=True):
+        super().__init__(CR, n, s, loss, Xs, ys, lr, beta0=beta0, K=K)
+        self.B = gc_cr_encoding(n, s, draws)
+        self.C = encoding_coefficients(self.B, self.c)
+        self.pipelined = pipelined
+
+    def evaluate(self):
+        if self.pipelined or self.t == 0:
+            return super().evaluate()
+        for i in range(self.n):                       # GC: all c partitions at beta^(t)
+            for l in range(self.c):
+                self.ring[i][l] = self.partition_grad(self.hold[i][l])
+                self.ring_step[i][l] = self.t
+
+    def coded(self, i):
+        """W_i's upload: sum_l c_{i,l} * its latest copy of g_{(i+l) mod n} (§V-A)."""
+        return sum(self.C[i][l] * self.ring[i][l] for l in range(self.c))
+
+    def decode(self, mask):
+        """(1/n) sum_m d_m(J) coded_{j_m} (§V-A; the 1/n is reading R14)."""
+        d = gc_decode_weights(self.B, mask)
+        g = np.zeros_like(self.beta)
+        for i in received_set(mask):
+            g = g + (d[i] / self.n) * self.coded(i)
+        return g
+
+    def step(self, mask):
+        d = gc_decode_weights(self.B, mask)
+        alpha = decoding_alpha(self.B, d, mask, self.c)
+        rec = super().step(mask)
+        if not self.pipelined:
+            rec["slot"] = -1
+            rec["eval_partition"] = [-1] * self.n
+        rec["coeff"] = d / self.n
+        rec["d"] = d
+        rec["alpha"] = alpha
+        rec["alpha_max"] = max(alpha.values())
+        rec["alpha_min"] = min(alpha.values())
+        return rec
+
+
+def run_mode(mode, scheme, n, s, loss, Xs, ys, lr, masks, beta0=None, K=1, record_loss=True, draws=None):
+    """run() for a training mode: "pgc", "is_sgd", "gc" (GC with FR placement,
+    or with CR placement and GC-CR's coefficients when scheme is CR) or
+    "naive_cr" (§V-A)."""
     if mode == "pgc":
         return run(scheme, n, s, loss, Xs, ys, lr, masks, beta0=beta0, K=K, record_loss=record_loss)
-    cls = {"is_sgd": ISSGDOracle, "gc": GCFROracle}[mode]
-    o = cls(n, s, loss, Xs, ys, lr, beta0=beta0, K=K)
+    if mode == "naive_cr" or (mode == "gc" and scheme == CR):
+        o = NaiveCROracle(n, s, loss, Xs, ys, lr, draws=draws, beta0=beta0, K=K, pipelined=mode == "naive_cr")
+    else:
+        cls = {"is_sgd": ISSGDOracle, "gc": GCFROracle}[mode]
+        o = cls(n, s, loss, Xs, ys, lr, beta0=beta0, K=K)
     out = []
     for mask in masks:
         lv = o.loss_value() if record_loss else None
