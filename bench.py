@@ -39,6 +39,7 @@ from paper_2607_20739_gb300 import workloads as W  # noqa: E402
 METRIC = "PGC steps/s & samples/s at 1 GB300; % of HBM (or bf16 TC) roofline"
 DEFAULT_WORKLOAD = "cr_n8_logistic_d1024"
 L2_BYTES = 129 * 2 ** 20
+GC_DRAWS_SEED = 2607          # seed of the GC-CR encoding draws (naive_cr, and gc on CR placement)
 
 
 def parse_args(argv=None):
@@ -49,7 +50,7 @@ def parse_args(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=W.WORKLOAD_ORDER)
     ap.add_argument("--seed", type=int, default=1)
-    ap.add_argument("--mode", default="pgc", choices=["pgc", "is_sgd", "gc"],
+    ap.add_argument("--mode", default="pgc", choices=["pgc", "is_sgd", "gc", "naive_cr"],
                     help="training scheme on the same kernels: PGC, or the IS-SGD / GC (FR) baselines")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0, help="budget of the oracle sample")
@@ -232,11 +233,15 @@ def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 
     S = {"FR": O.FR, "CR": O.CR}
     L = {"logistic": O.LOGISTIC, "lsq": O.LSQ, "softmax": O.SOFTMAX}
     Xf = [W.features_as_float(X, w.dtype) for X in Xs]
+    gc_cr = mode == "naive_cr" or (mode == "gc" and w.scheme == "CR")
     if mode == "pgc":
         o = O.PGCOracle(S[w.scheme], w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
+    elif gc_cr:
+        o = O.NaiveCROracle(w.n, w.s, L[w.loss], Xf, ys, w.lr, draws=W.make_gc_draws(w, GC_DRAWS_SEED), K=w.K,
+                            pipelined=mode == "naive_cr")
     else:
         o = {"is_sgd": O.ISSGDOracle, "gc": O.GCFROracle}[mode](w.n, w.s, L[w.loss], Xf, ys, w.lr, K=w.K)
-    inner = o if mode == "pgc" else o.inner
+    inner = o if mode == "pgc" or gc_cr else o.inner
     evals_per_step = w.n * (w.c if mode == "gc" else 1)
     t0 = time.perf_counter()
     inner.partition_grad(0)
@@ -335,6 +340,8 @@ def run_ours(args):
     stream = torch.cuda.Stream(device=dev)
     g = B.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream, mode=args.mode)
     g.load(Xs, ys)
+    if args.mode == "naive_cr" or (args.mode == "gc" and w.scheme == "CR"):
+        g.set_gc_encoding(W.make_gc_draws(w, GC_DRAWS_SEED))
     P = w.K * w.d
     gout = torch.empty(P, device=dev)
     wout = torch.empty(P, device=dev)

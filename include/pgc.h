@@ -36,6 +36,9 @@ extern "C" {
 #define PGC_ETIMEOUT (-7)  /* a bounded device-side wait gave up            */
 #define PGC_ESCRATCH (-8)  /* problem larger than pgc_gradient_noalloc's
                               fixed scratch                                 */
+#define PGC_ESINGULAR (-9) /* GC-CR: the draws leave a worker's encoding
+                              system singular, or the encoding cannot decode
+                              the straggler set                             */
 
 /* ---- enumerations (passed as int32) ------------------------------------ */
 /* Dataset placement, §III: FR needs c | n; CR places cyclically.          */
@@ -88,11 +91,23 @@ int pgc_create(pgc_ctx **out, int32_t n, int32_t s, int32_t scheme, int32_t loss
                                the master averages the n - s received gradients.
                                Needs scheme PGC_CR (the decode runs as CR with one
                                slot per worker, coefficient 1/(n - s)).             */
-#define PGC_MODE_GC     2   /* gradient coding with fractional repetition: every
-                               worker evaluates all c partitions of its group each
-                               step; the master decodes one coded gradient per group
-                               (1/n), which recovers (1/n) sum_k g_k exactly.  Needs
-                               scheme PGC_FR (GC-CR's coefficients are only cited). */
+#define PGC_MODE_GC     2   /* gradient coding (GC, §VI-A): every worker evaluates
+                               all c of its partitions each step.  PGC_FR: the
+                               master decodes one coded gradient per group (1/n),
+                               which recovers (1/n) sum_k g_k exactly.  PGC_CR:
+                               GC-CR (§V-A), worker W_j uploads
+                               sum_l c_{j,l} g_{(j+l) mod n} with the encoding of
+                               pgc_set_gc_encoding and the master applies the
+                               decode weights d_m(J) of the received set, times
+                               1/n: exact as well.  PGC_CR needs n <= 64.        */
+#define PGC_MODE_NAIVE_CR 3 /* the naive pipelined construction on cyclic
+                               repetition (§V-A): PGC-CR's rotation and stores
+                               (one partition evaluated per step), but W_j uploads
+                               sum_l c_{j,l} (its latest gradient of
+                               D_{(j+l) mod n}) and the master decodes with GC-CR's
+                               weights d_m(J), times 1/n.  Stale copies enter with
+                               the decoding coefficients alpha_{m,k} = d_m c_{j_m,l}
+                               (pgc_get_gc_decode).  Needs PGC_CR and n <= 64.   */
 
 /*
  * pgc_create_mode — pgc_create with a training scheme from PGC_MODE_*; the
@@ -103,6 +118,47 @@ int pgc_create(pgc_ctx **out, int32_t n, int32_t s, int32_t scheme, int32_t loss
 int pgc_create_mode(pgc_ctx **out, int32_t mode, int32_t n, int32_t s, int32_t scheme, int32_t loss,
                     int32_t dtype, int64_t d, int64_t K, const int64_t *rows, float lr,
                     const float *w0, void *stream);
+
+/*
+ * pgc_set_gc_encoding — GC-CR's encoding coefficients c_{j,l} (§V-A), for the
+ * modes that decode with them (PGC_MODE_NAIVE_CR; PGC_MODE_GC with PGC_CR).
+ * §V-A takes them from gradient coding's cyclic-repetition construction,
+ * which the device builds from the given random numbers: H = [draws |
+ * -(row sums of draws)] is s x n with H 1 = 0; worker W_j's row of the
+ * encoding matrix B is supported on partitions j..j+s (mod n), has
+ * c_{j,0} = B[j][j] = 1, and its other s entries solve
+ * H[:, {j+1..j+s}] x = -H[:, j] (fp64, partial pivoting).
+ *   draws : host array [s][n-1], row-major (for instance standard normal
+ *           draws); ignored when s = 0 (then B is the identity).
+ * Must be called before the first pgc_step of those modes (PGC_ESTATE
+ * otherwise); may be called again.  Not part of a checkpoint.  Errors:
+ * PGC_EINVAL (other mode, NULL or non-finite draws), PGC_ESINGULAR (a
+ * worker's system is singular; the context stays usable), PGC_ECUDA.
+ */
+int pgc_set_gc_encoding(pgc_ctx *ctx, const double *draws);
+
+/*
+ * pgc_get_gc_encoding — copy the encoding coefficients to host coeff[n][c]:
+ * coeff[j*c + l] = c_{j,l}, W_j's weight on its gradient of D_{(j+l) mod n}.
+ * Errors: PGC_EINVAL (other mode), PGC_ESTATE (not set), PGC_ECUDA.
+ */
+int pgc_get_gc_encoding(pgc_ctx *ctx, double *coeff);
+
+/*
+ * pgc_get_gc_decode — what the device derived at the last step of a GC-CR
+ * mode (§V-A): d (host [n], or NULL) = the decode weights d_j(J) solving
+ * sum_{j in J} d_j B[j] = 1 over the received set J (0 for stragglers), in
+ * fp64; alpha_range (host [2], or NULL) = the maximum and the minimum of the
+ * decoding coefficients alpha_{m,k} = d_m c_{j_m,l} over the received workers
+ * and the partitions each holds.  The decoded gradient is
+ * (1/n) sum_j d_j sum_l c_{j,l} store[j][l].  A straggler set the encoding
+ * cannot decode (sum_j d_j B[j] misses 1 by more than 1e-8 relative, or a
+ * pivot vanishes) leaves that step's beta unchanged and makes the call that
+ * reads the device status (pgc_step with host outputs, pgc_sync) return
+ * PGC_ESINGULAR; the context then takes no more steps.  Errors: PGC_EINVAL,
+ * PGC_ESTATE (no step yet), PGC_ECUDA.
+ */
+int pgc_get_gc_decode(pgc_ctx *ctx, double *d, double *alpha_range);
 
 /*
  * pgc_load_partitions — copy the n partitions into device memory (§III: the
@@ -214,7 +270,8 @@ int pgc_get_store_cols(pgc_ctx *ctx, int32_t worker, int32_t slot, int64_t col0,
  * pgc_get_decode — the decoding coefficients the device derived from the
  * last step's mask: coeff[i] (host [n]) = weight a_i of W_i's coded gradient
  * (§IV-A: 1/n for each FR group's representative; §V-B: 1/((n-s)c) for each
- * received CR worker; 0 otherwise).  Errors: PGC_ESTATE, PGC_ECUDA.
+ * received CR worker; GC-CR modes: d_i(J)/n; 0 otherwise).  Errors:
+ * PGC_ESTATE, PGC_ECUDA.
  */
 int pgc_get_decode(pgc_ctx *ctx, float *coeff);
 

@@ -24,7 +24,7 @@ if not os.path.exists(LIB_PATH):
 
 lib = C.CDLL(LIB_PATH)
 
-OK, EINVAL, EMASK, ESTATE, ENOMEM, ECUDA, ENOTSUP, ETIMEOUT, ESCRATCH = 0, -1, -2, -3, -4, -5, -6, -7, -8
+OK, EINVAL, EMASK, ESTATE, ENOMEM, ECUDA, ENOTSUP, ETIMEOUT, ESCRATCH, ESINGULAR = 0, -1, -2, -3, -4, -5, -6, -7, -8, -9
 FR, CR = 0, 1
 LOGISTIC, LSQ, SOFTMAX = 0, 1, 2
 F32, BF16 = 0, 1
@@ -32,8 +32,8 @@ F32, BF16 = 0, 1
 SCHEMES = {"FR": FR, "CR": CR}
 LOSSES = {"logistic": LOGISTIC, "lsq": LSQ, "softmax": SOFTMAX}
 DTYPES = {"f32": F32, "bf16": BF16}
-MODE_PGC, MODE_IS_SGD, MODE_GC = 0, 1, 2
-MODES = {"pgc": MODE_PGC, "is_sgd": MODE_IS_SGD, "gc": MODE_GC}
+MODE_PGC, MODE_IS_SGD, MODE_GC, MODE_NAIVE_CR = 0, 1, 2, 3
+MODES = {"pgc": MODE_PGC, "is_sgd": MODE_IS_SGD, "gc": MODE_GC, "naive_cr": MODE_NAIVE_CR}
 
 
 class StepInfo(C.Structure):
@@ -65,6 +65,9 @@ _sig = {
     "pgc_checkpoint_load": (C.c_int, [_vp, _vp, _i64]),
     "pgc_get_store_cols": (C.c_int, [_vp, _i32, _i32, _i64, _i64, C.POINTER(C.c_float)]),
     "pgc_get_decode": (C.c_int, [_vp, C.POINTER(C.c_float)]),
+    "pgc_set_gc_encoding": (C.c_int, [_vp, C.POINTER(C.c_double)]),
+    "pgc_get_gc_encoding": (C.c_int, [_vp, C.POINTER(C.c_double)]),
+    "pgc_get_gc_decode": (C.c_int, [_vp, C.POINTER(C.c_double), C.POINTER(C.c_double)]),
     "pgc_get_weights": (C.c_int, [_vp, C.POINTER(C.c_float)]),
     "pgc_set_weights": (C.c_int, [_vp, C.POINTER(C.c_float)]),
     "pgc_step_count": (C.c_int64, [_vp]),
@@ -257,6 +260,28 @@ class PGC:
         out = np.zeros(self.n, dtype=np.float32)
         _check(lib.pgc_get_decode(self._h, out.ctypes.data_as(C.POINTER(C.c_float))), "pgc_get_decode")
         return out
+
+    def set_gc_encoding(self, draws=None) -> None:
+        """GC-CR's encoding from the construction's draws [s][n-1] (§V-A)."""
+        p = None
+        if self.s > 0:
+            draws = np.ascontiguousarray(np.asarray(draws, dtype=np.float64).reshape(self.s, self.n - 1))
+            p = draws.ctypes.data_as(C.POINTER(C.c_double))
+        _check(lib.pgc_set_gc_encoding(self._h, p), "pgc_set_gc_encoding")
+
+    def gc_encoding(self) -> np.ndarray:
+        """Encoding coefficients c_{j,l}, shape [n][c]."""
+        out = np.zeros((self.n, self.c), dtype=np.float64)
+        _check(lib.pgc_get_gc_encoding(self._h, out.ctypes.data_as(C.POINTER(C.c_double))), "pgc_get_gc_encoding")
+        return out
+
+    def gc_decode(self):
+        """The last step's decode weights d_j(J) [n] and (max, min) of alpha_{m,k}."""
+        d = np.zeros(self.n, dtype=np.float64)
+        ar = np.zeros(2, dtype=np.float64)
+        _check(lib.pgc_get_gc_decode(self._h, d.ctypes.data_as(C.POINTER(C.c_double)),
+                                     ar.ctypes.data_as(C.POINTER(C.c_double))), "pgc_get_gc_decode")
+        return d, (float(ar[0]), float(ar[1]))
 
     def store_cols(self, worker: int, slot: int, col0: int, ncols: int) -> np.ndarray:
         """Columns [col0, col0 + ncols) of the flattened K*d stored gradient."""

@@ -148,6 +148,13 @@ struct pgc_ctx {
   int tcg_pairs = 0;         // co-resident CTA pairs of the gradient contraction
   alignas(64) unsigned char tmXq[128];   // X as the fused kernel's A part (box 64 x 128/NT)
   alignas(64) unsigned char tmRst[128];  // Rb as the fused kernel's output (box 64 x 32)
+  // GC-CR coding: the naive PGC-CR mode and GC with cyclic repetition (§V-A)
+  bool gc_weighted = false;    // decode with GC-CR's weights instead of PGC's slot totals
+  bool gc_ready = false;       // encoding coefficients set (pgc_set_gc_encoding)
+  double* gc_coeff = nullptr;  // [n][c] encoding coefficients c_{j,l}
+  double* gc_d = nullptr;      // [n + 2] the last step's d_j, then max and min alpha
+  double* gc_draws = nullptr;  // [s][n-1] the construction's draws (staging)
+  float* gc_wts = nullptr;     // [n][c] the last step's d_j c_{j,l} / n
   int64_t loss_chunk = 0;
   int loss_nblocks = 256;
   void* tables = nullptr;
@@ -190,6 +197,7 @@ int read_status(pgc_ctx* ctx) {
   if (e != cudaSuccess) return cuda_fail(ctx, e);
   if (h & kErrWaitTimeout) { ctx->broken = true; return PGC_ETIMEOUT; }
   if (h & kErrBadMask) { ctx->broken = true; return PGC_EMASK; }
+  if (h & kErrSingular) { ctx->broken = true; return PGC_ESINGULAR; }
   if (h) { ctx->broken = true; return PGC_ECUDA; }
   return PGC_OK;
 }
@@ -238,12 +246,30 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
     if (const char* env = std::getenv("PGC_ITEMS_PER_SM")) per_sm = std::max(1, std::atoi(env));
     const int64_t G = (int64_t)ctx->sm_count * per_sm;
     const int64_t min_rows = grad_rows_stage_rows(ctx->variant, ctx->ld, ctx->dtype);
+    // items of (nearly) one length L for every partition: the smallest L whose
+    // item count fits one wave of the grid, so that all CTAs finish together
+    // (items of unequal length leave the long ones to fewer CTAs at the end)
+    std::vector<int64_t> qe(nE), cap(nE);
+    int64_t mmax = 1;
+    for (int e = 0; e < nE; ++e) {
+      cap[e] = std::max<int64_t>(1, ph.e_rows[e] / min_rows);
+      mmax = std::max(mmax, ph.e_rows[e]);
+    }
+    auto count = [&](int64_t L) {
+      int64_t tot = 0;
+      for (int e = 0; e < nE; ++e) tot += std::min(cap[e], std::max<int64_t>(1, (ph.e_rows[e] + L - 1) / L));
+      return tot;
+    };
+    int64_t lo = 1, hi = mmax;                 // count(mmax) = nE: the fewest items possible
+    while (lo < hi) {
+      const int64_t mid = lo + (hi - lo) / 2;
+      if (count(mid) <= G) hi = mid; else lo = mid + 1;
+    }
+    for (int e = 0; e < nE; ++e) qe[e] = std::min(cap[e], std::max<int64_t>(1, (ph.e_rows[e] + lo - 1) / lo));
     ph.e_item0.push_back(0);
     for (int e = 0; e < nE; ++e) {
       const int64_t m = ph.e_rows[e];
-      int64_t q = (int64_t)std::llround((double)G * (double)m / (double)R);
-      q = std::max<int64_t>(q, 1);
-      q = std::min<int64_t>(q, std::max<int64_t>(1, m / min_rows));
+      const int64_t q = qe[e];
       for (int64_t i = 0; i < q; ++i) {
         const int64_t a = m * i / q, b = m * (i + 1) / q;
         WorkItem it;
@@ -364,7 +390,8 @@ void free_all(pgc_ctx* ctx) {
   for (cudaEvent_t ev : ctx->ev_pool) cudaEventDestroy(ev);
   ctx->ev_pool.clear();
   void* ptrs[] = {ctx->X, ctx->y, ctx->w, ctx->wb, ctx->store, ctx->U, ctx->gout, ctx->partials, ctx->Z,
-                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->tables, ctx->counters, ctx->Rb};
+                  ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->tables, ctx->counters, ctx->Rb,
+                  ctx->gc_coeff, ctx->gc_d, ctx->gc_draws, ctx->gc_wts};
   for (void* p : ptrs)
     if (p) cudaFree(p);
 }
@@ -404,6 +431,7 @@ const char* pgc_strerror(int32_t code) {
     case PGC_ENOTSUP: return "unsupported combination";
     case PGC_ETIMEOUT: return "a bounded device-side wait timed out";
     case PGC_ESCRATCH: return "problem too large for the fixed scratch of pgc_gradient_noalloc";
+    case PGC_ESINGULAR: return "GC-CR: singular encoding system, or a straggler set the encoding cannot decode";
     default: return "unknown status";
   }
 }
@@ -442,9 +470,12 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   *out = nullptr;
   int rc = check_nsc(scheme, n, s);
   if (rc) return rc;
-  if (mode != PGC_MODE_PGC && mode != PGC_MODE_IS_SGD && mode != PGC_MODE_GC) return PGC_EINVAL;
-  if (mode == PGC_MODE_IS_SGD && scheme != PGC_CR) return PGC_EINVAL;
-  if (mode == PGC_MODE_GC && scheme != PGC_FR) return PGC_EINVAL;
+  if (mode != PGC_MODE_PGC && mode != PGC_MODE_IS_SGD && mode != PGC_MODE_GC && mode != PGC_MODE_NAIVE_CR)
+    return PGC_EINVAL;
+  if ((mode == PGC_MODE_IS_SGD || mode == PGC_MODE_NAIVE_CR) && scheme != PGC_CR) return PGC_EINVAL;
+  // GC-CR's decode weights come from per-step fp64 solves on one warp
+  const bool gc_weighted = mode == PGC_MODE_NAIVE_CR || (mode == PGC_MODE_GC && scheme == PGC_CR);
+  if (gc_weighted && n > kGcMaxN) return PGC_ENOTSUP;
   if (!valid_loss(loss) || !valid_dtype(dtype) || d < 1 || !rows || !std::isfinite(lr)) return PGC_EINVAL;
   if (loss == PGC_SOFTMAX ? (K < 2 || K > 4096) : K != 1) return PGC_EINVAL;
   for (int k = 0; k < n; ++k)
@@ -455,6 +486,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   if (!ctx) return PGC_ENOMEM;
   // IS-SGD keeps one slot per worker (its own partition) and still ignores s stragglers
   ctx->mode = mode;
+  ctx->gc_weighted = gc_weighted;
   ctx->n = n; ctx->s = s; ctx->c = mode == PGC_MODE_IS_SGD ? 1 : s + 1;
   ctx->scheme = scheme; ctx->loss = loss; ctx->dtype = dtype;
   ctx->d = d; ctx->K = K; ctx->lr = lr;
@@ -498,6 +530,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
       const int box = rows_box_blocks(ldr, req);
       ctx->sk_box = box;
       if (const char* env = std::getenv("PGC_NO_ROWS_TAIL")) ctx->sk_tail = env[0] != '1';
+      if (gc_weighted) ctx->sk_tail = false;   // its fused decode is PGC's
       // the occupancy query first: it makes the runtime's context current,
       // which the tensor-map encoder (a driver call) needs
       const int nctas = slots >= 2 ? rows_max_ctas(ldr, slots) : 0;
@@ -528,7 +561,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     // needs quickly: the refreshed slot of every store, the other slot
     // totals and the stragglers' stores, about (owners + c + s c) P floats
     const double dec_bytes = (double)(ctx->owners + ctx->c + (double)s * ctx->c) * ctx->P * 4.0;
-    ctx->tail_mode = dec_bytes <= 512.0 * 1024.0 ? 2 : 1;
+    ctx->tail_mode = dec_bytes <= 512.0 * 1024.0 && !gc_weighted ? 2 : 1;
   }
 
   cudaError_t e = cudaGetDevice(&ctx->device);
@@ -625,6 +658,12 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   PGC_ALLOC(ctx->loss_out, sizeof(double));
   PGC_ALLOC(ctx->tables, tab.size());
   PGC_ALLOC(ctx->counters, (size_t)(n + 3) * sizeof(int));
+  if (gc_weighted) {
+    PGC_ALLOC(ctx->gc_coeff, (size_t)n * ctx->c * sizeof(double));
+    PGC_ALLOC(ctx->gc_d, (size_t)(n + 2) * sizeof(double));
+    PGC_ALLOC(ctx->gc_draws, (size_t)s * (n - 1) * sizeof(double));
+    PGC_ALLOC(ctx->gc_wts, (size_t)n * ctx->c * sizeof(float));
+  }
 
   cudaStream_t st = ctx->stream;
   e = cudaMemcpyAsync(ctx->tables, tab.data(), tab.size(), cudaMemcpyHostToDevice, st);
@@ -636,6 +675,8 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->coeff, 0, (size_t)n * sizeof(float), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->status, 0, sizeof(int), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(ctx->counters, 0, (size_t)(n + 3) * sizeof(int), st);
+  if (e == cudaSuccess && gc_weighted) e = cudaMemsetAsync(ctx->gc_wts, 0, (size_t)n * ctx->c * sizeof(float), st);
+  if (e == cudaSuccess && gc_weighted) e = cudaMemsetAsync(ctx->gc_d, 0, (size_t)(n + 2) * sizeof(double), st);
   if (e == cudaSuccess && w0)
     e = cudaMemcpy2DAsync(ctx->w, ctx->ld * sizeof(float), w0, d * sizeof(float), d * sizeof(float), K,
                           cudaMemcpyHostToDevice, st);
@@ -735,6 +776,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
              pgc_step_info* info) {
   if (!ctx || !mask) return PGC_EINVAL;
   if (!ctx->loaded || ctx->broken) return PGC_ESTATE;
+  if (ctx->gc_weighted && !ctx->gc_ready) return PGC_ESTATE;
   const int n = ctx->n, c = ctx->c;
   MaskBits bits;
   std::memset(&bits, 0, sizeof(bits));
@@ -792,7 +834,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     // in steady phases every evaluated partition has one store at slot o_t,
     // so the backward also forms U[o_t] = sum_e g_e (TMA reduce-add) and the
     // decode reads it instead of re-summing the stores
-    const bool u_red = ph.slot >= 0 && ph.ndest == 1;
+    const bool u_red = ph.slot >= 0 && ph.ndest == 1 && !ctx->gc_weighted;
     f.a_off = ph.d_f_aoff; f.total_tiles = ph.f_prefix.back();
     f.out_row0 = ph.d_f_outrow0; f.status = ctx->status; f.pdl = ctx->pdl ? 1 : 0;
     if (ctx->tcf) {
@@ -874,7 +916,14 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     PGC_CK(ctx, launch_commit(cm, st, ctx->pdl));
   }
   PGC_CK(ctx, record_event(ctx));
-  if (need_decode) {
+  if (need_decode && ctx->gc_weighted) {
+    // GC-CR: the step's decode weights (one CTA, fp64), then the weighted decode + SGD
+    GcWeightsArgs gw;
+    gw.n = n; gw.s = ctx->s; gw.c = c; gw.mask = bits; gw.coeff = ctx->gc_coeff; gw.d = ctx->gc_d;
+    gw.wts = ctx->gc_wts; gw.coeff_out = ctx->coeff; gw.alpha = ctx->gc_d + n; gw.status = ctx->status;
+    nl[PGC_KDECODE] = 2;
+    PGC_CK(ctx, launch_gc_decode(gw, dc, st, ctx->pdl, ctx->sm_count));
+  } else if (need_decode) {
     // K5+K6 decode + SGD
     nl[PGC_KDECODE] = 1;
     PGC_CK(ctx, launch_decode(dc, st, ctx->pdl, ctx->sm_count));
@@ -960,6 +1009,51 @@ int pgc_get_decode(pgc_ctx* ctx, float* coeff) {
   if (!ctx || !coeff) return PGC_EINVAL;
   if (!ctx->stepped || ctx->broken) return PGC_ESTATE;
   PGC_CK(ctx, cudaMemcpyAsync(coeff, ctx->coeff, (size_t)ctx->n * sizeof(float), cudaMemcpyDeviceToHost, ctx->stream));
+  return read_status(ctx);
+}
+
+int pgc_set_gc_encoding(pgc_ctx* ctx, const double* draws) {
+  if (!ctx || !ctx->gc_weighted) return PGC_EINVAL;
+  if (ctx->broken) return PGC_ESTATE;
+  const int n = ctx->n, s = ctx->s;
+  if (s > 0 && !draws) return PGC_EINVAL;
+  for (int64_t i = 0; i < (int64_t)s * (n - 1); ++i)
+    if (!std::isfinite(draws[i])) return PGC_EINVAL;
+  cudaStream_t st = ctx->stream;
+  if (s > 0)
+    PGC_CK(ctx, cudaMemcpyAsync(ctx->gc_draws, draws, (size_t)s * (n - 1) * sizeof(double), cudaMemcpyHostToDevice, st));
+  PGC_CK(ctx, launch_gc_encoding(ctx->gc_draws, n, s, ctx->gc_coeff, ctx->status, st));
+  int h = 0;
+  PGC_CK(ctx, cudaMemcpyAsync(&h, ctx->status, sizeof(int), cudaMemcpyDeviceToHost, st));
+  PGC_CK(ctx, cudaStreamSynchronize(st));
+  if (h == kErrSingular) {
+    // the draws leave some worker's system singular: keep the context usable
+    PGC_CK(ctx, cudaMemsetAsync(ctx->status, 0, sizeof(int), st));
+    PGC_CK(ctx, cudaStreamSynchronize(st));
+    ctx->gc_ready = false;
+    return PGC_ESINGULAR;
+  }
+  if (h) return read_status(ctx);
+  ctx->gc_ready = true;
+  return PGC_OK;
+}
+
+int pgc_get_gc_encoding(pgc_ctx* ctx, double* coeff) {
+  if (!ctx || !coeff || !ctx->gc_weighted) return PGC_EINVAL;
+  if (!ctx->gc_ready || ctx->broken) return PGC_ESTATE;
+  PGC_CK(ctx, cudaMemcpyAsync(coeff, ctx->gc_coeff, (size_t)ctx->n * ctx->c * sizeof(double), cudaMemcpyDeviceToHost,
+                              ctx->stream));
+  return read_status(ctx);
+}
+
+int pgc_get_gc_decode(pgc_ctx* ctx, double* d, double* alpha_range) {
+  if (!ctx || !ctx->gc_weighted || (!d && !alpha_range)) return PGC_EINVAL;
+  if (!ctx->stepped || ctx->broken) return PGC_ESTATE;
+  if (d)
+    PGC_CK(ctx, cudaMemcpyAsync(d, ctx->gc_d, (size_t)ctx->n * sizeof(double), cudaMemcpyDeviceToHost, ctx->stream));
+  if (alpha_range)
+    PGC_CK(ctx, cudaMemcpyAsync(alpha_range, ctx->gc_d + ctx->n, 2 * sizeof(double), cudaMemcpyDeviceToHost,
+                                ctx->stream));
   return read_status(ctx);
 }
 

@@ -12,6 +12,7 @@ enum : int {
   kErrWaitTimeout = 1,   // a bounded mbarrier wait gave up
   kErrBadMask = 2,       // the decode kernel saw a mask with popcount != s
   kErrBadShape = 4,      // a kernel was launched with an impossible shape
+  kErrSingular = 8,      // GC-CR: the draws cannot encode, or the straggler set cannot be decoded
 };
 
 // A contiguous row range of one evaluated partition, processed by one CTA.
@@ -112,6 +113,24 @@ struct CommitArgs {
 cudaError_t launch_commit(const CommitArgs& a, cudaStream_t st, bool pdl = false);
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st, bool pdl, int sm_count);
+
+// ---- GC-CR coding: the naive pipelined construction and GC-CR (§V-A) -------
+constexpr int kGcMaxN = 64;   // workers of the GC-CR modes (one-warp fp64 solves)
+struct GcWeightsArgs {
+  int n, s, c;
+  MaskBits mask;
+  const double* coeff;      // [n][c] encoding coefficients c_{j,l}
+  double* d;                // [n] decode weights d_j(J), 0 for stragglers
+  float* wts;               // [n][c] d_j c_{j,l} / n, applied to store[j][l]
+  float* coeff_out;         // [n] d_j / n, the weight of W_j's coded gradient
+  double* alpha;            // [2] max and min of alpha_{m,k} = d_m c_{j_m,l}
+  int* status;
+};
+// Encoding coefficients [n][c] from draws [s][n-1] (device); one launch.
+cudaError_t launch_gc_encoding(const double* draws, int n, int s, double* coeff, int* status, cudaStream_t st);
+// The step's decode weights (one CTA), then decode + SGD over the stores
+// (programmatic dependent of the weights kernel when pdl is set).
+cudaError_t launch_gc_decode(const GcWeightsArgs& w, const DecodeArgs& a, cudaStream_t st, bool pdl, int sm_count);
 
 // ---- generic softmax gradient on CUDA cores --------------------------------
 // logits Z[r][k] = sum_j W[k][j] x_r[j] for the rows of each evaluated

@@ -188,6 +188,12 @@ def draw_delays(w: Workload, steps: int, seed: int) -> np.ndarray:
     raise ValueError(w.delays)
 
 
+def make_gc_draws(w: Workload, seed: int) -> np.ndarray:
+    """float64 [s, n-1] standard normal draws: the random numbers of GC-CR's
+    cyclic-repetition encoding (§V-A), passed to both sides as an input."""
+    return np.random.default_rng(seed).standard_normal((w.s, w.n - 1))
+
+
 def make_masks(w: Workload, steps: int, seed: int) -> np.ndarray:
     """uint8 [steps, n]; 1 marks the s workers with the largest delay that step."""
     D = draw_delays(w, steps, seed)

@@ -36,7 +36,7 @@ def test_mode_parity_with_oracle(libpgc, cuda, name):
 
 def test_mode_scheme_pairs_are_checked(libpgc, cuda):
     w = WL["fr_n4_logistic_d64"]
-    for mode, scheme in (("is_sgd", "FR"), ("gc", "CR"), (7, "CR")):
+    for mode, scheme in (("is_sgd", "FR"), ("naive_cr", "FR"), (7, "CR")):
         with pytest.raises(libpgc.PGCError) as ei:
             libpgc.PGC(scheme, w.n, w.s, w.loss, w.dtype, w.d, rows=w.rows(), lr=w.lr, mode=mode)
         assert ei.value.code == libpgc.EINVAL
