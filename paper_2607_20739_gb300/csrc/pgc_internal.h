@@ -235,8 +235,9 @@ struct TcGradParams {
 constexpr int kTcGradMaxRun = 8;   // partitions per unit at most
 // Clusters of two that fit at once (0: the kernel cannot be launched).
 int tc_grad_max_pairs();
-cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, const TcGradParams& p, int npairs,
-                           cudaStream_t st);
+// tmS: the stores [owners * c][K][ld] fp32, box 32 x 32 x 1 (written by TMA)
+cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, const void* tmS, const TcGradParams& p,
+                           int npairs, cudaStream_t st);
 
 // ---- tensor-core logits GEMM with the softmax residual in its epilogue ------
 // (tc_softmax.cu) for every 128-row tile {first X row, first R row, valid

@@ -51,6 +51,14 @@ __device__ __forceinline__ void tma_reduce_add_3d_hint(const CUtensorMap* tm, co
       "r"(x), "r"(y), "r"(z), "r"(smem_u32(src)), "l"(policy)
       : "memory");
 }
+__device__ __forceinline__ void tma_store_3d_hint(const CUtensorMap* tm, const void* src, int x, int y, int z,
+                                                  uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.tile.bulk_group.L2::cache_hint [%0, {%1, %2, %3}], [%4], %5;" ::"l"(
+          tm),
+      "r"(x), "r"(y), "r"(z), "r"(smem_u32(src)), "l"(policy)
+      : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }

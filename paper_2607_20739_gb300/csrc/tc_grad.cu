@@ -49,11 +49,6 @@ __host__ __device__ constexpr GradSmem grad_smem() {
                   kGS * (kGA + kGB) + kGEpi * kGBox + 16 * 8};
 }
 
-__device__ __forceinline__ void st_global_v4_hint(float* dst, float4 v, uint64_t pol) {
-  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(dst), "f"(v.x),
-               "f"(v.y), "f"(v.z), "f"(v.w), "l"(pol)
-               : "memory");
-}
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 
 // stage 8 values (columns 8 qt .. 8 qt + 7) of this lane's row into its
@@ -71,7 +66,7 @@ __device__ __forceinline__ void stage_quarter(uint8_t* box, int lane, int qt, co
 // the slot total in them and reads TMEM 16 columns at a time.
 __global__ void __launch_bounds__(kGThreads, 1)
 tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmX,
-               const __grid_constant__ CUtensorMap tmU, TcGradParams p) {
+               const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmS, TcGradParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr GradSmem L = grad_smem();
@@ -230,23 +225,20 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
             if (rows_exist) stage_quarter(box, lane, qt, g);
           }
           if (rows_exist) {
-            // read the box back transposed (lane: 16-byte chunk lane % 8 of
-            // rows 4 it + lane / 8) and write whole 128-byte rows
+            // the box goes to every store keeping the copy by TMA (rows past
+            // the class count are outside the map and dropped); it is
+            // rewritten only after these copies have read it
+            fence_proxy_async_smem();
             __syncwarp();
-            const uint64_t pol = policy_evict_first();
-            const int cc = lane & 7;
-            for (int k = 0; k < p.ndest; ++k) {
-              const int dd = dl[k];
-              if (dd < 0) continue;
-              float* dst = p.store + (int64_t)dd * p.P + (int64_t)row0 * p.ld + n0 + ch * 32 + cc * 4;
-#pragma unroll 1
-              for (int it = 0; it < 8; ++it) {
-                const int rr = 4 * it + (lane >> 3);
-                const float4 v = reinterpret_cast<const float4*>(box + rr * 128)[cc ^ (rr & 7)];
-                if (row0 + rr < p.m_limit) st_global_v4_hint(dst + (int64_t)rr * p.ld, v, pol);
+            if (lane == 0) {
+              const uint64_t pol = policy_evict_first();
+              for (int k = 0; k < p.ndest; ++k) {
+                const int dd = dl[k];
+                if (dd >= 0) tma_store_3d_hint(&tmS, box, n0 + ch * 32, row0, dd, pol);
               }
+              bulk_commit();
             }
-            __syncwarp();
+            pending = true;
           }
         }
         tc_fence_before();
@@ -323,8 +315,8 @@ int tc_grad_max_pairs() {
   return mp;
 }
 
-cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, const TcGradParams& p, int npairs,
-                           cudaStream_t st) {
+cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, const void* tmS, const TcGradParams& p,
+                           int npairs, cudaStream_t st) {
   if (p.nunits <= 0) return cudaSuccess;
   if (npairs < 1) return cudaErrorInvalidValue;
   const size_t smem = grad_smem_bytes();
@@ -345,11 +337,12 @@ cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, co
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.pdl ? 2 : 1;
-  CUtensorMap a, b, u;
+  CUtensorMap a, b, u, w;
   std::memcpy(&a, tmR, sizeof(CUtensorMap));
   std::memcpy(&b, tmX, sizeof(CUtensorMap));
   std::memcpy(&u, tmU, sizeof(CUtensorMap));
-  return cudaLaunchKernelEx(&cfg, tc_grad_kernel, a, b, u, p);
+  std::memcpy(&w, tmS, sizeof(CUtensorMap));
+  return cudaLaunchKernelEx(&cfg, tc_grad_kernel, a, b, u, w, p);
 }
 
 }  // namespace pgc

@@ -154,3 +154,22 @@ def test_gc_cr_errors(libpgc, cuda):
     g.step(mask, grad, None)
     assert np.isfinite(grad).all()
     g.close()
+
+
+EDGE = {
+    # the largest n the GC-CR modes take (one-warp fp64 solves over 64 rows)
+    "naive_cr_n64_max": ("naive_cr", WL["cr_n8_logistic_d1024"].replace(n=64, s=3, m=9, d=40, lr=0.05), 5),
+    # s = 0: B is the identity, every decode weight 1, the step is DGD
+    "naive_cr_s0": ("naive_cr", WL["cr_n8_logistic_d1024"].replace(n=5, s=0, m=30, d=48, lr=0.05), 3),
+    # c = n: every worker holds every partition, one coded gradient decodes
+    "naive_cr_c_equals_n": ("naive_cr", WL["cr_n8_logistic_d1024"].replace(n=4, s=3, m=25, d=36, lr=0.05), 6),
+    "gc_cr_c_equals_n": ("gc", WL["cr_n8_logistic_d1024"].replace(n=3, s=2, m=25, d=36, lr=0.05), 3),
+    # one row per partition and d = 1
+    "naive_cr_one_row_d1": ("naive_cr", WL["cr_n64_lsq_d16384"].replace(n=6, s=2, m=1, d=1, lr=0.05), 4),
+}
+
+
+@pytest.mark.parametrize("name", list(EDGE))
+def test_gc_cr_edge_cases(libpgc, cuda, name):
+    mode, w, T = EDGE[name]
+    run_and_compare(libpgc, w, T, mode=mode)
