@@ -313,7 +313,7 @@ __device__ void consumer_commit(const GradRowsArgs& a, const Smem& sm, int e, in
 
 __device__ void consumer_decode(const GradRowsArgs& a, const Smem& sm, int tid) {
   if (tid < 32) write_coeffs_warp(a.dec, tid);
-  decode_columns(a.dec, *sm.plan, tid, kNT);
+  decode_columns(a.dec, *sm.plan, 0, a.dec.P / 4, tid, kNT);
 }
 
 // Item end, consumer side, called by all 8 warps at the same stage.

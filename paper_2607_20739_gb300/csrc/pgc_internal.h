@@ -308,12 +308,12 @@ struct RowsArgs {
   int box_blocks;           // 64-feature blocks per TMA copy (divides ld / 64)
   int* status;
   int pdl;
-  // Fused tail (tail = 1): after a grid barrier every CTA commits a share of
-  // the (partition, column) pairs (ordered sum of the partition's items,
-  // times e_scale, into each destination store), then after a second
-  // barrier decodes and updates w (dec) over a share of the columns.  The
-  // grid must be co-resident (one CTA per SM); counters[0..2] are zero
-  // between steps (the last CTA resets them).
+  // Fused tail (tail = 1): after a grid barrier every CTA commits, for its
+  // slice of the float4 columns, every evaluated partition (ordered sum of the
+  // partition's items, times e_scale, into each destination store), then
+  // after a CTA barrier decodes and updates w (dec) over the same columns.
+  // The grid must be co-resident (one CTA per SM); counters[0] and
+  // counters[2] are zero between steps (the last CTA resets them).
   int tail = 0;
   int nE = 0;
   const int32_t* e_item0 = nullptr;  // [nE + 1]

@@ -24,11 +24,11 @@
 //      in a partition, and frees the slot with tcgen05.commit.
 // No data leaves the pair before the end of a run; then the eight warps write
 // the run's G^T halves into one partial (one item per pair and partition).
-// With the fused tail the same grid then commits (after a grid barrier: every
-// CTA sums a share of the partitions' items in item order, scales by 1/m_e and
-// writes the stores) and decodes (after a second barrier: coefficients from
-// the mask, decode and SGD over a share of the columns); otherwise separate
-// commit and decode kernels follow.
+// With the fused tail the same grid then commits and decodes: after a grid
+// barrier each CTA sums, for its slice of the columns, every partition's items
+// in item order, scales by 1/m_e and writes the stores, then (after a CTA
+// barrier) decodes and updates the same columns with the coefficients it
+// derived from the mask; otherwise separate commit and decode kernels follow.
 // Every wait is bounded; the TMEM allocation is released on every path.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -489,15 +489,20 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
   tc_fence_after();
   if (a.tail && !*cta_err) {
     // ---- fused tail: commit, then decode + SGD --------------------------------
+    // After one grid barrier (every partial written) each CTA commits every
+    // evaluated partition for its own slice of the float4 columns and then
+    // decodes that slice: a column's decode reads only that column of the
+    // stores and slot totals, all written by this CTA, so a CTA barrier
+    // stands in for a second grid barrier.
     if (warp == 0) derive_plan_warp(a.dec, plan, lane);   // needs only the mask
-    const int64_t gt = (int64_t)blockIdx.x * blockDim.x + threadIdx.x, GT = (int64_t)gridDim.x * blockDim.x;
     const int64_t P4 = a.P / 4;
+    const int64_t q0 = P4 * blockIdx.x / gridDim.x, q1 = P4 * (blockIdx.x + 1) / gridDim.x, nq = q1 - q0;
     bool ok = grid_barrier(a.counters, a.status, &bar_flag);   // every partial is written
     if (ok) {
       const float4* src = reinterpret_cast<const float4*>(a.partials);
-      for (int64_t x = gt; x < (int64_t)a.nE * P4; x += GT) {
-        const int e = (int)(x / P4);
-        const int64_t p = x - (int64_t)e * P4;
+      for (int64_t x = threadIdx.x; x < (int64_t)a.nE * nq; x += blockDim.x) {
+        const int e = (int)(x / nq);
+        const int64_t p = q0 + (x - (int64_t)e * nq);
         const int i0 = a.e_item0[e], i1 = a.e_item0[e + 1];
         float4 acc = f4zero();
         for (int it = i0; it < i1; it += 8) {
@@ -514,16 +519,13 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
           if (dst >= 0) reinterpret_cast<float4*>(a.store)[(int64_t)dst * P4 + p] = acc;
         }
       }
-      ok = grid_barrier(a.counters + 1, a.status, &bar_flag);   // every store is committed
-    }
-    if (ok) {
+      __syncthreads();                   // this CTA's stores are visible to all its threads
       if (blockIdx.x == 0 && warp == 0) write_coeffs_warp(a.dec, lane);
-      decode_columns(a.dec, plan, (int)gt, (int)GT);
+      decode_columns(a.dec, plan, q0, q1, (int)threadIdx.x, (int)blockDim.x);
       __syncthreads();
       // the last CTA out resets the counters for the next step
       if (threadIdx.x == 0 && atomic_add_acq_rel(a.counters + 2, 1) == (int)gridDim.x - 1) {
         a.counters[0] = 0;
-        a.counters[1] = 0;
         a.counters[2] = 0;
         __threadfence();
       }

@@ -149,10 +149,11 @@ __device__ __forceinline__ void store_outputs(const DecodeArgs& a, int64_t p, fl
   }
 }
 
-// Decode + SGD with every column handled by one thread and no barriers, for
-// one CTA covering a small P.  When the counts fit the unrolled bounds all
-// loads of a column are issued back to back; otherwise plain loops.
-__device__ __forceinline__ void decode_columns(const DecodeArgs& a, const DecodePlan& pl, int tid, int nthr) {
+// Decode + SGD of the float4 columns [q0, q1), every column handled by one
+// thread (tid of nthr) and no barriers.  When the counts fit the unrolled
+// bounds all loads of a column are issued back to back; otherwise plain loops.
+__device__ __forceinline__ void decode_columns(const DecodeArgs& a, const DecodePlan& pl, int64_t q0, int64_t q1,
+                                               int tid, int nthr) {
   constexpr int kMaxO = 8, kMaxC = 4, kMaxD = 4;
   const int64_t P4 = a.P / 4;
   const int c = a.c;
@@ -161,7 +162,7 @@ __device__ __forceinline__ void decode_columns(const DecodeArgs& a, const Decode
   const float4* store = reinterpret_cast<const float4*>(a.store);
   float4* U = reinterpret_cast<float4*>(a.U);
   const bool small = a.owners <= kMaxO && c <= kMaxC && ndev <= kMaxD && a.slot >= 0 && !a.u_ready;
-  for (int64_t p = tid; p < P4; p += nthr) {
+  for (int64_t p = q0 + tid; p < q1; p += nthr) {
     float4 V = f4zero(), D = f4zero();
     if (small) {
       float4 u[kMaxO], o4[kMaxC], dv[kMaxD][kMaxC];
