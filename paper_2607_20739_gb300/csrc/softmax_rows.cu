@@ -505,12 +505,14 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         const int64_t p = q0 + (x - (int64_t)e * nq);
         const int i0 = a.e_item0[e], i1 = a.e_item0[e + 1];
         float4 acc = f4zero();
-        for (int it = i0; it < i1; it += 8) {
-          float4 v[8];
+        // a partition has about (pairs / partitions) + 1 items: one batch of
+        // loads in flight covers it
+        for (int it = i0; it < i1; it += 16) {
+          float4 v[16];
 #pragma unroll
-          for (int u = 0; u < 8; ++u) v[u] = it + u < i1 ? __ldcg(src + (int64_t)(it + u) * P4 + p) : f4zero();
+          for (int u = 0; u < 16; ++u) v[u] = it + u < i1 ? __ldcg(src + (int64_t)(it + u) * P4 + p) : f4zero();
 #pragma unroll
-          for (int u = 0; u < 8; ++u) acc = f4add(acc, v[u]);
+          for (int u = 0; u < 16; ++u) acc = f4add(acc, v[u]);
         }
         const float sc = a.e_scale[e];
         acc = make_float4(acc.x * sc, acc.y * sc, acc.z * sc, acc.w * sc);

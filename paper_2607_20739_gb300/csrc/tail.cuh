@@ -47,7 +47,7 @@ __device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void commit_block(const float* partials, int64_t P, int i0, int i1, float scale,
                                              const int32_t* dest, int ndest, float* store, int tid, int nthr) {
-  constexpr int kB = 16;          // partials loaded per batch
+  constexpr int kB = 20;          // partials loaded per batch (one item per SM: 152 / 8 = 19 at n = 8)
   const int64_t P4 = P / 4;
   const float4* src = reinterpret_cast<const float4*>(partials);
   for (int64_t p = tid; p < P4; p += nthr) {
