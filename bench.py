@@ -121,7 +121,7 @@ def kernel_label(w: W.Workload, single: bool, dom: int) -> str:
         return "tc_gemm_kernel, logits X W^T (tcgen05, 2-CTA clusters)"
     if w.loss == "softmax" and w.dtype == "bf16" and w.K <= 16:
         if -(-w.d // 128) * 128 <= 3072:
-            return "softmax_rows_kernel (whole 16-row tiles per CTA, one pass over X)"
+            return "softmax_rows_kernel (16-row tiles split by features over CTA pairs, one pass over X; whole step)"
         return "softmax_smallk_kernel (8-CTA clusters, one pass over X)"
     if w.loss == "softmax":
         return "CUDA-core softmax gradient kernels"
