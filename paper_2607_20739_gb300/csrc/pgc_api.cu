@@ -62,6 +62,8 @@ struct Phase {
   std::vector<int32_t> sk_tiles;
   int sk_items = 0;
   int32_t* d_sk_tiles = nullptr;
+  std::vector<int32_t> sk_cuts;   // whole-row variant: tile range of each CTA pair
+  int32_t* d_sk_cuts = nullptr;
   // device copies
   WorkItem* d_items = nullptr;
   int32_t* d_e_item0 = nullptr;
@@ -298,10 +300,42 @@ void build_phase(pgc_ctx* ctx, Phase& ph, int slot) {
       }
     // runs per cluster (whole-row variant: per CTA pair)
     const int64_t T = (int64_t)te.size(), nc = ctx->sk_rows ? ctx->sk_nc / 2 : ctx->sk_nc;
+    std::vector<int64_t> cut(nc + 1);
+    for (int64_t cl = 0; cl <= nc; ++cl) cut[cl] = T * cl / nc;
+    if (ctx->sk_rows) {
+      // each tile costs 1 and each run that starts inside a pair's range
+      // kRowsDrainTiles more (the previous run's drain stalls the pair); the
+      // smallest largest cost whose greedy fill covers every tile
+      // (PGC_ROWS_DRAIN_TILES overrides the charge)
+      int64_t D = kRowsDrainTiles;
+      if (const char* env = std::getenv("PGC_ROWS_DRAIN_TILES")) D = std::max(0, std::atoi(env));
+      auto fill = [&](int64_t C) {
+        int64_t i = 0;
+        for (int64_t p = 0; p < nc; ++p) {
+          cut[p] = i;
+          int64_t cost = 0;
+          while (i < T) {
+            const int64_t add = 1 + ((i > cut[p] && te[i] != te[i - 1]) ? D : 0);
+            if (cost + add > C) break;
+            cost += add;
+            ++i;
+          }
+        }
+        cut[nc] = i;
+        return i;
+      };
+      int64_t lo = (T + nc - 1) / nc, hi = lo + D * nE + 1;
+      while (lo < hi) {
+        const int64_t mid = lo + (hi - lo) / 2;
+        if (fill(mid) >= T) hi = mid; else lo = mid + 1;
+      }
+      fill(lo);
+      for (int64_t cl = 0; cl <= nc; ++cl) ph.sk_cuts.push_back((int32_t)cut[cl]);
+    }
     std::vector<int32_t> items_of(nE, 0);
     int item = 0;
     for (int64_t cl = 0; cl < nc; ++cl) {
-      const int64_t a = T * cl / nc, b = T * (cl + 1) / nc;
+      const int64_t a = cut[cl], b = cut[cl + 1];
       for (int64_t i = a; i < b; ++i) {
         const bool first = i == a || te[i] != te[i - 1];
         const bool last = i == b - 1 || te[i] != te[i + 1];
@@ -592,7 +626,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   std::vector<uint8_t> tab;
   size_t off = 0;
   std::vector<size_t> offs;
-  constexpr int kTabs = 19;
+  constexpr int kTabs = 20;
   for (auto& ph : ctx->phases) {
     offs.push_back(align_up(off, 16)); put(tab, off, ph.items);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.e_item0);
@@ -613,6 +647,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     offs.push_back(align_up(off, 16)); put(tab, off, ph.sk_tiles);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.q_tiles);
     offs.push_back(align_up(off, 16)); put(tab, off, ph.g_units);
+    offs.push_back(align_up(off, 16)); put(tab, off, ph.sk_cuts);
   }
   // loss chunks (softmax): {row0, rows, 0} per chunk
   std::vector<int64_t> ldesc;
@@ -714,6 +749,7 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     ph.d_sk_tiles = reinterpret_cast<int32_t*>(base + o[16]);
     ph.d_q_tiles = reinterpret_cast<int32_t*>(base + o[17]);
     ph.d_g_units = reinterpret_cast<int32_t*>(base + o[18]);
+    ph.d_sk_cuts = reinterpret_cast<int32_t*>(base + o[19]);
   }
   ctx->loss_desc = nullptr;
   if (!ldesc.empty()) ctx->loss_desc = reinterpret_cast<int64_t*>(base + ldesc_off);
@@ -877,6 +913,7 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     need_commit = false;
   } else if (ctx->sk_rows) {
     RowsArgs a;
+    a.pair_t0 = ph.d_sk_cuts;
     a.tiles = reinterpret_cast<const int4*>(ph.d_sk_tiles); a.ntiles = (int)(ph.sk_tiles.size() / 4);
     a.K = (int)ctx->K; a.y = static_cast<const int32_t*>(ctx->y); a.wb = ctx->wb;
     a.partials = ctx->partials; a.P = ctx->P; a.ld = ctx->ld; a.nslots = ctx->sk_slots; a.box_blocks = ctx->sk_box;

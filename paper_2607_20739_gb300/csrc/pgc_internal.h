@@ -292,10 +292,15 @@ cudaError_t launch_softmax_smallk(const void* tmX, const void* tmW, const SmallK
 // one per half of the features) takes tiles [ntiles p / Np, ntiles (p + 1) / Np).
 // partials[item][K][ld] receives the unscaled gradient sums of the run.
 constexpr int kRowsTileRows = 16;
+// A run (one partition's tiles) that starts inside a CTA pair's range stalls
+// the pair's logits warps while the previous run drains: about this many
+// tiles' time, charged when the host splits the tiles over the pairs.
+constexpr int kRowsDrainTiles = 4;
 constexpr int64_t kRowsMaxLd = 3072;       // the forward keeps a warp's W^T slice in registers
 constexpr int kRowsMaxSlots = 8;
 constexpr uint32_t kRowsSmemBudget = 227 * 1024 - 1024;   // a little static shared memory beside it
 struct RowsArgs {
+  const int32_t* pair_t0;   // [pairs + 1]: CTA pair p takes tiles [pair_t0[p], pair_t0[p + 1])
   const int4* tiles;
   int ntiles;
   int K;

@@ -18,10 +18,15 @@
 //      memory, add the two blocks in rank order (so both CTAs form the same
 //      R) and form R = softmax(Z) - onehot(y) (zero past K and past the
 //      partition's rows) in bf16, in the no-swizzle K-major operand layout;
-//   3. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
-//      the 16 rows; A = the resident half tile read MN-major) into a TMEM
+//   3. the same eight warps copy the half tile, transposed, into tensor memory
+//      (one lane per feature, two rows per 32-bit column: the K-major A
+//      operand of the gradient MMA) and release the slot, so a slot is held
+//      only for its load, the logits and the copy, not for the exchange of
+//      step 2; kNA copies (and R blocks) rotate;
+//   4. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
+//      the 16 rows; A = the tile's copy in tensor memory, B = R) into a TMEM
 //      accumulator of the CTA's half of G^T that spans the pair's run of tiles
-//      in a partition, and frees the slot with tcgen05.commit.
+//      in a partition; its commit frees the copy and the R block.
 // No data leaves the pair before the end of a run; then the eight warps write
 // the run's G^T halves into one partial (one item per pair and partition).
 // With the fused tail the same grid then commits and decodes: after a grid
@@ -53,7 +58,13 @@ constexpr int kRThreads = 64 + 32 * kFw + 32 * kNRes;
 constexpr int kMaxKs = (int)(kRowsMaxLd / kPairCtas / (16 * kFw));
 constexpr uint32_t kZp = kRR * 16 * 4;   // a 16 x 16 fp32 block of partial logits
 constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16)
-constexpr int kTmemCols = 256;           // G^T half: ld / 256 slices of 16 columns
+constexpr int kNA = 3;                   // tiles whose gradient MMA may be pending (TMEM copies, R blocks)
+constexpr int kTmemCols = 512;           // G^T half, then the kNA copies of a tile
+constexpr uint32_t kAccCols = 192;       // G^T half: ld / 256 slices of 16 columns at the largest ld
+constexpr uint32_t kAStride = 96;        // a copy: ld / 256 slices of 8 columns (16 rows of bf16)
+static_assert(kRowsMaxLd / kPairCtas / 128 * 16 <= (int)kAccCols, "G^T half fits its columns");
+static_assert(kRowsMaxLd / kPairCtas / 128 * 8 <= (int)kAStride, "a tile copy fits its columns");
+static_assert(kAccCols + kNA * kAStride <= (uint32_t)kTmemCols, "tensor memory holds G^T and the copies");
 
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t layout) {
   uint64_t d = 0;
@@ -82,6 +93,37 @@ __device__ __forceinline__ void mma16816(float (&c)[4], uint32_t a0, uint32_t a1
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& a0, uint32_t& a1, uint32_t& a2, uint32_t& a3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3)
+               : "r"(addr));
+}
+// 16 lanes x 8 columns from the warp: thread t writes lanes t/4 and t/4 + 8,
+// columns 2 (t % 4) and 2 (t % 4) + 1 (the layout of an mma.sync accumulator)
+__device__ __forceinline__ void tmem_st_16x256b(uint32_t taddr, uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3) {
+  asm volatile("tcgen05.st.sync.aligned.16x256b.x1.b32 [%0], {%1,%2,%3,%4};" ::"r"(taddr), "r"(r0), "r"(r1), "r"(r2),
+               "r"(r3)
+               : "memory");
+}
+// K position of tile row r in the gradient MMA: the tensor-memory copy puts
+// row pair p (rows 2p, 2p + 1) in column 2p (p < 4) or 2 (p - 4) + 1, so R
+// is laid out with the same order of its K rows
+__device__ __forceinline__ int k_of_row(int r) {
+  const int p = r >> 1;
+  return 2 * (p < 4 ? 2 * p : 2 * p - 7) + (r & 1);
+}
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// D (+)= A B with A in tensor memory (K-major, one row per lane), B in shared memory
+__device__ __forceinline__ void umma_ta_fresh(uint32_t tmem_d, uint32_t tmem_a, uint64_t db, uint32_t idesc) {
+  asm volatile("tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, 0;" ::"r"(tmem_d), "r"(tmem_a), "l"(db),
+               "r"(idesc)
+               : "memory");
+}
+__device__ __forceinline__ void umma_ta_acc(uint32_t tmem_d, uint32_t tmem_a, uint64_t db, uint32_t idesc) {
+  asm volatile("tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, 1;" ::"r"(tmem_d), "r"(tmem_a), "l"(db),
+               "r"(idesc)
+               : "memory");
 }
 // shared::cta address -> the same offset in CTA `rank` of the cluster
 __device__ __forceinline__ uint32_t mapa_u32(uint32_t addr, uint32_t rank) {
@@ -161,18 +203,18 @@ __device__ bool grid_barrier(int* ctr, int* status, int* flag) {
 
 // Shared memory of a CTA: slots of its half tile, two sets (tile parity) of
 // the forward warps' partial logits (the fused tail's decode plan reuses
-// them), two blocks for the other CTA's partial, R blocks, barriers.
+// them), two blocks for the other CTA's partial, kNA R blocks, barriers.
 struct RowsSmem {
   uint32_t slot_bytes, zpart, zpeer, rblk, bars, total;
 };
-constexpr int kRowsBars = 3 * kRowsMaxSlots + 8 + 4;
+constexpr int kRowsBars = 2 * kRowsMaxSlots + 3 * kNA + 8 + 4;
 __host__ __device__ static RowsSmem rows_smem(int64_t ld, int nslots) {
   RowsSmem s;
   s.slot_bytes = (uint32_t)(kRR * (ld / kPairCtas) * 2);
   s.zpart = (uint32_t)nslots * s.slot_bytes;
   s.zpeer = s.zpart + 2 * kFw * kZp;
   s.rblk = s.zpeer + 2 * kZp;
-  s.bars = s.rblk + (uint32_t)nslots * kRb;
+  s.bars = s.rblk + (uint32_t)kNA * kRb;
   s.total = s.bars + kRowsBars * 8 + 16;
   return s;
 }
@@ -191,9 +233,11 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
   uint8_t* rblk = sm + L.rblk;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.bars);
   uint64_t* full = bars;                          // [S] half tile landed
-  uint64_t* empty = bars + kRowsMaxSlots;         // [S] the tile's MMAs are done (slot, R block free)
-  uint64_t* rready = bars + 2 * kRowsMaxSlots;    // [S] R block written
-  uint64_t* zready = bars + 3 * kRowsMaxSlots;    // [2] every forward warp's partial written
+  uint64_t* empty = bars + kRowsMaxSlots;         // [S] the forward warps are done with the half tile
+  uint64_t* rready = bars + 2 * kRowsMaxSlots;    // [kNA] R block written
+  uint64_t* a_full = rready + kNA;                // [kNA] the tile's copy in tensor memory written
+  uint64_t* a_empty = a_full + kNA;               // [kNA] the tile's MMAs are done (copy, R block free)
+  uint64_t* zready = a_empty + kNA;               // [2] every forward warp's partial written
   uint64_t* zfree = zready + 2;                   // [2] the residual warp has read them
   uint64_t* zpeer_full = zready + 4;              // [2] the other CTA's block arrived
   uint64_t* zpeer_empty = zready + 6;             // [2] the other CTA has read this CTA's block
@@ -206,18 +250,21 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
   const int rank = (int)cluster_rank();
   const int64_t ldh = a.ld / kPairCtas;          // features of this CTA
   const int nmt = (int)(ldh / 128);              // 128-feature M slices of the backward
-  // this pair's tiles: [T p / Np, T (p + 1) / Np)
-  const int pair = (int)blockIdx.x / kPairCtas, npairs = (int)gridDim.x / kPairCtas;
-  const int t0 = (int)((int64_t)a.ntiles * pair / npairs);
-  const int t1 = (int)((int64_t)a.ntiles * (pair + 1) / npairs);
+  // this pair's tiles (split on the host)
+  const int pair = (int)blockIdx.x / kPairCtas;
+  const int t0 = a.pair_t0[pair], t1 = a.pair_t0[pair + 1];
   const int n = t1 - t0;
 
   if (threadIdx.x == 0) {
     *cta_err = 0;
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
-      mbar_init(&rready[s], 1);
+      mbar_init(&empty[s], kFw);
+    }
+    for (int b = 0; b < kNA; ++b) {
+      mbar_init(&rready[b], 1);
+      mbar_init(&a_full[b], kFw);
+      mbar_init(&a_empty[b], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&zready[b], kFw);
@@ -268,32 +315,28 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     }
   } else if (warp == 1 && lane == 0) {
     // ---- backward MMAs: G^T[f][k] += sum_r X[r][f] R[r][k] ------------------
-    constexpr uint32_t id_bwd = idesc_bf16_f32(128, 16, true, false);
+    constexpr uint32_t id_bwd = idesc_bf16_f32(128, 16, false, false);
     bool ok = true;
     int run = 0;
     for (int i = 0; i < n && ok; ++i) {
-      const int s = i % S;
+      const int ab = i % kNA;
       const int4 tl = a.tiles[t0 + i];
       const bool first = (tl.w & 1) || i == 0, last = (tl.w & 2) || i == n - 1;
-      if (!mbar_wait(&full[s], (i / S) & 1, a.status) || !mbar_wait(&rready[s], (i / S) & 1, a.status)) {
+      if (!mbar_wait(&a_full[ab], (i / kNA) & 1, a.status) || !mbar_wait(&rready[ab], (i / kNA) & 1, a.status)) {
         ok = false;
         break;
       }
       if (first && run > 0 && !mbar_wait(acc_empty, (run - 1) & 1, a.status)) { ok = false; break; }
       tc_fence_after();
-      const uint32_t xs = smem_u32(sm + (size_t)s * L.slot_bytes);
-      const uint64_t db = sdesc(smem_u32(rblk + s * kRb), 256, 128, 0);
-      // slice mt: two 64-feature blocks kBlk apart, the K = 16 rows two 8-row
-      // groups 1 KB apart; slices 2 kBlk apart (the address field counts
-      // 16-byte units)
-      const uint64_t da0 = sdesc(xs, kBlk, 1024, 2);
-      constexpr uint64_t kStep = (2 * kBlk) >> 4;
+      const uint64_t db = sdesc(smem_u32(rblk + ab * kRb), 256, 128, 0);
+      // slice mt: its 128 features x 16 rows are columns kAccCols + ab kAStride + 8 mt ..
+      const uint32_t ta = tmem + kAccCols + (uint32_t)ab * kAStride;
       if (first) {
-        for (int mt = 0; mt < nmt; ++mt) umma_bf16_fresh(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)mt * kStep, db, id_bwd);
+        for (int mt = 0; mt < nmt; ++mt) umma_ta_fresh(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), db, id_bwd);
       } else {
-        for (int mt = 0; mt < nmt; ++mt) umma_bf16_acc(tmem + (uint32_t)(mt * 16), da0 + (uint64_t)mt * kStep, db, id_bwd);
+        for (int mt = 0; mt < nmt; ++mt) umma_ta_acc(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), db, id_bwd);
       }
-      umma_commit(&empty[s]);
+      umma_commit(&a_empty[ab]);
       if (last) {
         umma_commit(acc_full);
         ++run;
@@ -305,14 +348,13 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     // Two warps, for the even and the odd tiles (every buffer and barrier of
     // the exchange is per tile parity), so one tile's exchange with the other
     // CTA overlaps the next tile's.  lane: row lane / 2, classes 8 (lane & 1)
-    // .. + 7.  The R block of slot s is free again once the tile's half was
-    // loaded (its full wait, through the forward warps' zready, implies the
-    // slot's previous MMAs completed).
+    // .. + 7.  The R block i % kNA is written once tile i - kNA's MMAs have
+    // read it (a_empty).
     const int r = lane >> 1, kh = (lane & 1) * 8;
     const uint32_t peer = (uint32_t)(rank ^ 1);
     bool ok = true;
     for (int i = warp - kRWarp; i < n && ok; i += kNRes) {
-      const int s = i % S, b = i & 1;
+      const int b = i & 1;
       const int4 tl = a.tiles[t0 + i];
       const bool valid = r < tl.y;
       const int lab = valid ? a.y[tl.x + r] : -1;        // fetched before the waits
@@ -372,16 +414,20 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       }
       sum += __shfl_xor_sync(0xffffffffu, sum, 1);
       const float inv = 1.0f / sum;
-      uint8_t* blk = rblk + s * kRb;
+      if (i >= kNA && !__all_sync(0xffffffffu, mbar_wait(&a_empty[i % kNA], ((i / kNA) - 1) & 1, a.status))) {
+        ok = false;
+        break;
+      }
+      uint8_t* blk = rblk + (i % kNA) * kRb;
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         const int k = kh + c;
         const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
-        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, r)) = __float2bfloat16_rn(v);
+        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, k_of_row(r))) = __float2bfloat16_rn(v);
       }
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&rready[s]);
+      if (lane == 0) mbar_arrive(&rready[i % kNA]);
     }
     if (!ok) atomicExch(cta_err, 1);
   } else if (warp >= 2) {
@@ -407,8 +453,45 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       }
     // ldmatrix row of this lane: matrix m = lane / 8 (rows 8 (m & 1) .., features 8 (m >> 1) ..)
     const int lr = ((lane >> 3) & 1) * 8 + (lane & 7), lk = (lane >> 4) * 8;
+    // The half tile j, transposed, into tensor memory as the gradient MMA's A
+    // operand: this warp writes lane quarter q (features 32 q .. of each
+    // 128-feature slice) of the slices of parity h; then slot j % S is
+    // released.  The copy of tile j - kNA must have been read by its MMAs.
+    // ldmatrix.trans of four 8 x 8 blocks (rows 0-7 / 8-15 x features fb ..
+    // fb + 7 / fb + 8 .. fb + 15) gives thread t rows 2 (t % 4), 2 (t % 4) + 1
+    // of each row half of features t / 4 and 8 + t / 4 (row pairs t % 4 and
+    // 4 + t % 4), stored as columns 2 (t % 4) and 2 (t % 4) + 1 of lanes t / 4
+    // and t / 4 + 8 (k_of_row gives R the same order of its K rows).
+    auto copy_tile = [&](int j) -> bool {
+      if (j >= kNA && !__all_sync(0xffffffffu, mbar_wait(&a_empty[j % kNA], ((j / kNA) - 1) & 1, a.status)))
+        return false;
+      tc_fence_after();
+      const int q = warp & 3, h = (warp - 2) >> 2;
+      const uint32_t xj = smem_u32(sm + (size_t)(j % S) * L.slot_bytes);
+      const uint32_t ta = tmem + ((uint32_t)(q * 32) << 16) + kAccCols + (uint32_t)(j % kNA) * kAStride;
+      const int mi = lane >> 3, mr = ((mi & 1) << 3) + (lane & 7);
+      for (int mt = h; mt < nmt; mt += 2) {
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const int f = mt * 128 + q * 32 + hh * 16 + ((mi >> 1) << 3);
+          const uint32_t ad = xj + (uint32_t)((f >> 6) * kBlk + mr * 128 + ((((f & 63) >> 3) ^ (mr & 7)) << 4));
+          uint32_t v0, v1, v2, v3;
+          ldsm_x4_trans(ad, v0, v1, v2, v3);
+          tmem_st_16x256b(ta + ((uint32_t)(hh * 16) << 16) + (uint32_t)(mt * 8), v0, v1, v2, v3);
+        }
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&a_full[j % kNA]);
+        mbar_arrive(&empty[j % S]);
+      }
+      return true;
+    };
     bool ok = true;
     int run = 0;
+    int pending = -1;
     for (int i = 0; i < n; ++i) {
       const int s = i % S, b = i & 1;
       const int4 tl = a.tiles[t0 + i];
@@ -452,6 +535,19 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       *reinterpret_cast<float2*>(zp + (g + 8) * 16 + 8 + 2 * tq) = make_float2(c1[2], c1[3]);
       __syncwarp();
       if (lane == 0) mbar_arrive(&zready[b]);
+      // the previous tile's copy waits until this tile's logits are handed
+      // over, so that the logits do not wait for tile i - kNA's MMAs; the last
+      // tile of a run is copied at once (its drain needs its MMAs)
+      if (pending >= 0) {
+        if (!copy_tile(pending)) { ok = false; break; }
+        pending = -1;
+      }
+      if (!last) {
+        pending = i;
+      } else if (!copy_tile(i)) {
+        ok = false;
+        break;
+      }
       if (last) {
         // end of the pair's run in a partition: this CTA's G^T slices -> its
         // half of the run's partial
@@ -535,10 +631,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
   }
   if (warp == 1) {
     // after a failure, wait (bounded) for the last commit before releasing TMEM
-    if (*cta_err && lane == 0 && n > 0) {
-      const int s = (n - 1) % S;
-      mbar_wait(&empty[s], ((n - 1) / S) & 1, a.status);
-    }
+    if (*cta_err && lane == 0 && n > 0) mbar_wait(&a_empty[(n - 1) % kNA], ((n - 1) / kNA) & 1, a.status);
     __syncwarp();
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"((uint32_t)kTmemCols)
