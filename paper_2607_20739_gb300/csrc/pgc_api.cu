@@ -902,7 +902,6 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
     b.units = reinterpret_cast<const int4*>(ph.d_g_units); b.nunits = (int)(ph.g_units.size() / 4);
     b.nk = ph.d_b_nk; b.a_off = ph.d_b_aoff; b.b_off = ph.d_b_boff;
     b.scale = ph.d_e_scale; b.dest = ph.d_e_dest; b.ndest = ph.ndest; b.m_limit = (int)ctx->K;
-    b.store = ctx->store; b.ld = ctx->ld; b.P = ctx->P;
     b.u_reduce = u_red ? 1 : 0; b.u_slot = ph.slot;
     b.status = ctx->status; b.pdl = ctx->pdl ? 1 : 0;
     PGC_CK(ctx, launch_tc_grad(ctx->tmR, ctx->tmXm, ctx->tmUo, ctx->tmSo, b, ctx->tcg_pairs, st));

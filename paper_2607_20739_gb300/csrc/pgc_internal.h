@@ -222,10 +222,7 @@ struct TcGradParams {
   const int* b_off;         // [nbatch] first X row of the batch
   const float* scale;       // [nbatch] 1/m_e
   const int32_t* dest;      // [nbatch * ndest] store index or -1
-  int ndest;
-  float* store;             // [slots][K][ld]
-  int64_t ld;               // row pitch of a store (floats)
-  int64_t P;                // K * ld: one store slot
+  int ndest;                // destinations: the stores, through the tmS tensor map
   int m_limit;              // classes that exist (K); rows past it are not written
   int u_reduce;
   int u_slot;
