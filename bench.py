@@ -219,6 +219,51 @@ class ClockSampler:
 # the fp64 oracle on the host cores (cpu_baseline and --impl reference)
 # ---------------------------------------------------------------------------
 
+# workloads whose oracle is also timed on one thread
+ONE_THREAD_WORKLOADS = ("fr_n4_logistic_d64", "cr_n8_logistic_d1024")
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.machine()
+
+
+def time_oracle_one_thread(w: W.Workload, seed: int, mode: str, budget_s: float):
+    """time_oracle in a child process whose BLAS and OpenMP pools have one
+    thread (the variables take effect only before numpy loads its BLAS).
+    Returns (steps/s, sample description) or None."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = ("import json, bench; from paper_2607_20739_gb300 import workloads as W; "
+            f"w = W.WORKLOADS[{w.name!r}]; Xs, ys = W.make_partitions(w, {seed}, threads=1); "
+            f"m = W.make_masks(w, 64, {seed + 1000}); "
+            f"v, k, el, d = bench.time_oracle(w, Xs, ys, m, {budget_s}, mode={mode!r}); "
+            "print(json.dumps([v, d]))")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True,
+                           timeout=max(120.0, 20 * budget_s))
+    except subprocess.TimeoutExpired:
+        return None
+    if r.returncode != 0 or not r.stdout.strip():
+        return None
+    v, d = json.loads(r.stdout.strip().splitlines()[-1])
+    return v, d
+
+
 def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 2, mode: str = "pgc"):
     """Steady steps/s of the oracle as it stands, and what was timed.
 
@@ -431,7 +476,12 @@ def run_ours(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, k, el, desc = time_oracle(w, Xs, ys, masks, args.cpu_seconds, mode=args.mode)
         cpu = {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
-               "sample": desc + "; fp64 numpy, BLAS threads = all cores"}
+               "sample": desc + "; fp64 numpy, BLAS threads = all cores", "cpu_model": cpu_model()}
+        if w.name in ONE_THREAD_WORKLOADS:
+            one = time_oracle_one_thread(w, args.seed, args.mode, min(8.0, args.cpu_seconds))
+            if one is not None:
+                cpu["value_1thread"] = one[0]
+                cpu["sample_1thread"] = one[1] + "; fp64 numpy, one thread"
     g.close()
 
     # ---- simulated wall clock of a step (the paper's time per step, PGC vs
@@ -501,7 +551,7 @@ def run_reference(args):
         "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
                    "rows_per_partition": w.m, "mode": args.mode},
         "cpu_baseline": {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": desc},
+                         "sample": desc, "cpu_model": cpu_model()},
         "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
