@@ -17,6 +17,10 @@ What each pin checks, and the passage that fixes it:
 * ``pin_cr_unbiased`` — eq. cr-unbiased (§V-B): the mean of the decoded
   gradient over all C(n, s) masks equals (1/(nc)) sum_{i,j} g_i^{s(t,i,j)}.
 
+* ``test_lsq_converges_to_the_normal_equations`` — least squares with equal
+  partitions: DGD and PGC-FR (stale copies, §IV-A) converge to the full-data
+  least-squares solution, solved directly with numpy.linalg.lstsq.
+
 ``test_planted_*`` plant a mistake in the oracle (monkeypatched, on the CPU)
 and check that at least one pin catches it.
 """
@@ -323,3 +327,31 @@ def test_planted_straggler_skips_evaluation(monkeypatch):
     monkeypatch.setattr(O.PGCOracle, "step", bad_step)
     with pytest.raises(AssertionError):
         pin_cr_fullsum(5, 2)
+
+
+# ---------------------------------------------------------------------------
+# Long-run sanity against a direct solve: least squares with equal partition
+# sizes has the full-data least-squares solution as its only stationary point
+# (sum_k X_k^T (X_k beta - y_k) = 0).  DGD (c = 1) converges to it; so does
+# PGC-FR, whose stale copies all equal the current gradient at a fixed point,
+# where the decode is (1/n) sum_k g_k = 0 (§IV-A; the theorem's geometric
+# convergence for a small enough eta).
+# ---------------------------------------------------------------------------
+
+def _normal_equations_solution(Xs, ys):
+    X = np.concatenate(Xs)
+    y = np.concatenate(ys)
+    return np.linalg.lstsq(X, y, rcond=None)[0]
+
+
+@pytest.mark.parametrize("scheme,s,lr,T", [(O.CR, 0, 0.2, 1500), (O.FR, 0, 0.2, 1500), (O.FR, 1, 0.1, 3000),
+                                           (O.FR, 3, 0.05, 6000)])
+def test_lsq_converges_to_the_normal_equations(scheme, s, lr, T):
+    n, m, d = 4, 6, 5
+    Xs, ys = _parts(n, m, d, loss=O.LSQ, seed=11)
+    o = O.PGCOracle(scheme, n, s, O.LSQ, Xs, ys, lr)
+    masks = [[1 if (i - t) % n < s else 0 for i in range(n)] for t in range(T)]
+    for mask in masks:
+        o.step(mask)
+    ref = _normal_equations_solution(Xs, ys)
+    np.testing.assert_allclose(o.beta, ref, rtol=0, atol=1e-9 * (1 + np.abs(ref).max()))
