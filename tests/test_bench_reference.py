@@ -1,7 +1,8 @@
-"""The reference arm of bench.py (the fp64 oracle on the host cores) prints
+"""bench.py on the CPU.  The reference arm (the fp64 oracle on the host cores) prints
 one JSON line with the fields the bench contract requires: the same metric,
 unit and direction as the GPU arm, its own e2e with no host-device traffic,
-and a cpu_baseline describing the run (kind oracle, cores, sample, CPU)."""
+and a cpu_baseline describing the run (kind oracle, cores, sample, CPU).  The
+roofline numerators of the five workloads match their shapes."""
 
 import json
 import os
@@ -41,3 +42,28 @@ def test_reference_line_fields(capsys, monkeypatch, mode):
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+# Algorithmic work per steady step of the five workloads, written out from
+# their shapes (X and labels of the distinct evaluated partitions read once;
+# the tensor-core contraction's 2 rows d K flops): the numerators of every
+# roofline fraction bench.py reports.
+EXPECTED_WORK = {
+    "fr_n4_logistic_d64": ("hbm", 2 * 256 * (64 * 4 + 4)),                  # FR: n/c = 2 partitions
+    "cr_n8_logistic_d1024": ("hbm", 8 * 8192 * (1024 * 4 + 4)),              # 268,697,600 B
+    "fr_n32_softmax_k10": ("hbm", 8 * 4096 * (3072 * 2 + 4)),                # 201,457,664 B
+    "cr_n64_lsq_d16384": ("hbm", 64 * 2048 * (16384 * 4 + 4)),               # 8,590,458,880 B
+    "cr_n128_softmax_k1000": ("tensor", 2.0 * 128 * 1024 * 4096 * 1000),      # 1.074 TFLOP per contraction
+}
+
+
+@pytest.mark.parametrize("name", list(EXPECTED_WORK))
+def test_roofline_numerators(name):
+    from paper_2607_20739_gb300 import workloads as W
+    bound, units, unit, peak = bench.roofline_model(W.WORKLOADS[name], {"hbm_gbs": 6784.8,
+                                                                        "bf16_tflops_sustained": 1718.2})
+    want_bound, want_units = EXPECTED_WORK[name]
+    assert bound == want_bound
+    assert units == pytest.approx(want_units, rel=0, abs=0.5)
+    assert peak == (6784.8 if bound == "hbm" else 1718.2)
+    assert unit == ("GB/s" if bound == "hbm" else "TFLOP/s")
