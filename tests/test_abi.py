@@ -27,8 +27,9 @@ def test_every_declared_symbol_is_exported(libpgc, root_dir):
 
 
 def test_strerror_covers_codes(libpgc):
-    for code in range(0, -9, -1):
+    for code in range(0, -10, -1):
         assert libpgc.lib.pgc_strerror(code)
+    assert b"GC-CR" in libpgc.lib.pgc_strerror(libpgc.ESINGULAR)
     assert b"unknown" in libpgc.lib.pgc_strerror(-99)
 
 
@@ -82,3 +83,29 @@ def test_null_context_calls(libpgc):
     assert L.pgc_sync(None) == libpgc.EINVAL
     assert L.pgc_step_count(None) == -1
     assert L.pgc_schedule(0, 4, 1, -1, None, None) == libpgc.EINVAL
+
+
+def _create_mode(lib, mode, n=4, s=1, scheme=1, loss=0, dtype=0, d=8, K=1):
+    h = C.c_void_p()
+    r = (C.c_int64 * n)(*([3] * n))
+    rc = lib.lib.pgc_create_mode(C.byref(h), mode, n, s, scheme, loss, dtype, d, K, r, C.c_float(0.1), None, None)
+    assert not h.value
+    return rc
+
+
+@pytest.mark.parametrize("mode,scheme,n,s,code", [
+    (7, 1, 4, 1, "EINVAL"),          # unknown mode
+    (1, 0, 4, 1, "EINVAL"),          # IS-SGD needs CR
+    (3, 0, 4, 1, "EINVAL"),          # naive PGC-CR needs CR
+    (3, 1, 65, 2, "ENOTSUP"),        # the GC-CR modes stop at n = 64
+    (2, 1, 65, 2, "ENOTSUP"),        # GC on CR placement uses the same decode weights
+])
+def test_create_mode_rejects_before_any_cuda_call(libpgc, mode, scheme, n, s, code):
+    assert _create_mode(libpgc, mode, n=n, s=s, scheme=scheme) == getattr(libpgc, code)
+
+
+def test_gc_cr_calls_on_a_null_context(libpgc):
+    L = libpgc.lib
+    assert L.pgc_set_gc_encoding(None, None) == libpgc.EINVAL
+    assert L.pgc_get_gc_encoding(None, None) == libpgc.EINVAL
+    assert L.pgc_get_gc_decode(None, None, None) == libpgc.EINVAL
