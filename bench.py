@@ -471,6 +471,20 @@ def run_ours(args):
     e2e_s = max_over_ranks(e2e_s, world, dev)
     e2e_value = world * e2e_steps / e2e_s
 
+    # ---- the GC-CR modes' decoding coefficients alpha_{m,k} (§V-A): their
+    # range, read after each of some untimed steps ------------------------
+    alpha = None
+    if args.mode == "naive_cr" or (args.mode == "gc" and w.scheme == "CR"):
+        amax, amin, big = -float("inf"), float("inf"), 0
+        na = min(200, len(mptr))
+        for t in range(na):
+            g.step(mptr[t], None, None, info=False)
+            _, (hi, lo) = g.gc_decode()
+            amax, amin = max(amax, hi), min(amin, lo)
+            big += int(max(abs(hi), abs(lo)) > 100.0)
+        alpha = {"max": amax, "min": amin, "steps": na, "steps_with_abs_over_100": big,
+                 "note": "alpha_{m,k} = d_m(J) c_{j_m,l} derived on the device each step (untimed steps)"}
+
     # ---- cpu baseline (rank 0, N = 1 only) -------------------------------
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -525,6 +539,8 @@ def run_ours(args):
         "simulated_wall_clock": sim,
         "clocks": clocks,
     }
+    if alpha is not None:
+        line["decoding_coefficients"] = alpha
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
