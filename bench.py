@@ -137,14 +137,41 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
 
 
+def _strip_comments(src: str) -> str:
+    """C/C++ source without its // and /* */ comments (string and character
+    literals kept), so that a comment-only edit leaves the hash unchanged."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        ch = src[i]
+        if ch in "\"'":
+            j = i + 1
+            while j < n and src[j] != ch:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(ch)
+            i += 1
+    return "".join(out)
+
+
 def kernel_source_hash() -> str:
+    """Hash of the kernel and host sources under csrc/ without comments, runs
+    of whitespace counted as one space: the recorded DRAM traffic stays valid
+    across comment-only edits."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_20739_gb300", "csrc")
     for f in sorted(os.listdir(csrc)):
         if f.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, f), "rb") as fh:
+            with open(os.path.join(csrc, f), encoding="utf-8") as fh:
                 h.update(f.encode())
-                h.update(fh.read())
+                h.update(" ".join(_strip_comments(fh.read()).split()).encode())
     return h.hexdigest()[:16]
 
 

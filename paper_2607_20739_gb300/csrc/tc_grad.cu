@@ -14,12 +14,13 @@
 // warp 1 issues tcgen05.mma (M = 128 classes, N = 256 features, K = 16 rows)
 // into one of two TMEM accumulators.  Eight epilogue warps (two per TMEM lane
 // quarter, 128 columns each) drain the other, 32 x 32 blocks at a time: a
-// block is written row-per-lane into the warp's swizzled scratch, read back
-// transposed and stored as whole 128-byte rows (st.global, evict-first: the
-// stores are only read back for stragglers), so no store waits on another;
-// each thread also keeps its row's share of the run's sum in registers, added
-// into U[o_t] with one TMA reduce-add per block at the end of the run.  So U
-// costs one reduce per run instead of one per partition.
+// block is written row-per-lane into the warp's 128-byte-swizzled box, which
+// one lane sends by TMA tensor store (evict-first: the stores are only read
+// back for stragglers) into every store that keeps the partition; the box is
+// rewritten once those copies have read it.  Each thread also keeps its row's
+// share of the run's sum in registers, added into U[o_t] with one TMA
+// reduce-add per block at the end of the run.  So U costs one reduce per run
+// instead of one per partition.
 // Every wait is bounded; the TMEM allocation is released on every path.
 #include <cuda.h>
 #include <cudaTypedefs.h>

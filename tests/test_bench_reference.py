@@ -67,3 +67,19 @@ def test_roofline_numerators(name):
     assert units == pytest.approx(want_units, rel=0, abs=0.5)
     assert peak == (6784.8 if bound == "hbm" else 1718.2)
     assert unit == ("GB/s" if bound == "hbm" else "TFLOP/s")
+
+
+def test_source_hash_ignores_comments_only(tmp_path, monkeypatch):
+    d = tmp_path / "paper_2607_20739_gb300" / "csrc"
+    d.mkdir(parents=True)
+    f = d / "k.cu"
+    f.write_text('// header\n__global__ void k(int* p) { p[0] = 1; /* one */ }\nconst char* s = "a//b";\n')
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h0 = bench.kernel_source_hash()
+    f.write_text('// header, reworded\n// over two lines\n__global__ void k(int* p) {\n  p[0] = 1;  // one\n}\n'
+                 'const char* s = "a//b";\n')
+    assert bench.kernel_source_hash() == h0
+    f.write_text('__global__ void k(int* p) { p[0] = 2; }\nconst char* s = "a//b";\n')
+    assert bench.kernel_source_hash() != h0
+    f.write_text('__global__ void k(int* p) { p[0] = 1; }\nconst char* s = "a/*b";\n')
+    assert bench.kernel_source_hash() != h0          # a comment marker inside a string is code
