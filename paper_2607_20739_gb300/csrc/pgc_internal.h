@@ -210,7 +210,8 @@ cudaError_t launch_softmax_bf16(const float* Z, uint16_t* Rb, int64_t Kpad, int6
 // ---- tensor-core gradient contraction (tc_grad.cu) -------------------------
 // G_e = scale_e R_e^T X_e for the runs of partitions in `units`
 // ({class pair tile mp, feature tile nt, first batch, batches}), written into
-// the stores [slot][K][ld] at every dest of the batch; with u_reduce each
+// the stores [slot][K][ld] at every dest of the batch (TMA tensor stores
+// through tmS); with u_reduce each
 // run's sum is also added (TMA reduce-add, fp32 box 32 x 32 x 1) into
 // U [c][K][ld] at u_slot.  R is read as MN-major A (box 64 x 64), X as
 // MN-major B (box 64 x 64).
@@ -285,8 +286,10 @@ cudaError_t launch_softmax_smallk(const void* tmX, const void* tmW, const SmallK
 
 // ---- softmax with few classes, whole rows per CTA pair (softmax_rows.cu) ---
 // tiles[i] = {first global X row, rows (<= kRowsTileRows), item, flags: 1 first / 2 last
-// tile of a pair's run in one partition}; pair p of Np (clusters of two CTAs,
-// one per half of the features) takes tiles [ntiles p / Np, ntiles (p + 1) / Np).
+// tile of a pair's run in one partition}; pair p (a cluster of two CTAs, one
+// per half of the features) takes tiles [pair_t0[p], pair_t0[p + 1]), a split
+// made on the host that charges kRowsDrainTiles for each run starting inside
+// a pair's range.
 // partials[item][K][ld] receives the unscaled gradient sums of the run.
 constexpr int kRowsTileRows = 16;
 // A run (one partition's tiles) that starts inside a CTA pair's range stalls
