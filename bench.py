@@ -1,20 +1,24 @@
 #!/usr/bin/env python
-"""Throughput of the PGC hot path on GB300: one JSON line on stdout.
+"""Throughput of the PGC hot path on one GB300: one JSON line on stdout.
 
 A "step" is one ``pgc_step`` call: every scheduled per-partition gradient,
 the gradient-store commit, and the decode fused with the SGD update, over the
 workload's resident partitions.  ``value`` is steady-state steps/s measured
-with CUDA events on the library's stream (inputs resident in HBM), max over
-ranks.  ``e2e`` is the same metric through the Python API with host buffers:
-the straggler mask goes host->device and the decoded gradient and the new
-parameters come back device->host every step.
+with CUDA events on the library's stream (inputs resident in HBM).  ``e2e`` is
+the same metric through the Python API with host buffers: the straggler mask
+goes host->device and the decoded gradient and the new parameters come back
+device->host every step.
 
-  python bench.py [--workload NAME] [--steps K] [--warmup W] [--gpus N]
-  python bench.py --impl reference ...   # the fp64 CPU oracle, same workload
+  python bench.py [--steps K] [--warmup W]          # headline + every workload
+  python bench.py --workload NAME [--override k=v]  # one workload only
+  python bench.py --impl reference ...              # the fp64 CPU oracle
 
-With --gpus N > 1 (under torchrun) each rank runs an independent replica of
-the whole simulated cluster (the path keeps all n workers on one GPU), so the
-scaling is weak and ``value`` is the sum over ranks.
+By default the headline line is the largest workload, cr_n128_softmax_k1000
+(CR, n=128, s=7, softmax K=1000, d=4096), timed over exactly K steps, and
+``per_workload`` carries the same fields for the other four workloads,
+measured in the same invocation.  The simulated cluster lives on one GPU:
+there is no multi-GPU form, so ``--gpus`` other than 1, or a launch with
+several ranks, stops with an error before any CUDA call.
 """
 
 from __future__ import annotations
@@ -37,7 +41,7 @@ sys.path.insert(0, ROOT)
 from paper_2607_20739_gb300 import workloads as W  # noqa: E402
 
 METRIC = "PGC steps/s & samples/s at 1 GB300; % of HBM (or bf16 TC) roofline"
-DEFAULT_WORKLOAD = "cr_n8_logistic_d1024"
+HEADLINE_WORKLOAD = "cr_n128_softmax_k1000"   # the largest workload that fits one GPU
 L2_BYTES = 129 * 2 ** 20
 GC_DRAWS_SEED = 2607          # seed of the GC-CR encoding draws (naive_cr, and gc on CR placement)
 
@@ -48,7 +52,9 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=None)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=W.WORKLOAD_ORDER)
+    ap.add_argument("--workload", default=None, choices=W.WORKLOAD_ORDER,
+                    help="measure this workload only (default: the headline workload, then every other one)")
+    ap.add_argument("--no-per-workload", action="store_true", help="measure the headline workload only")
     ap.add_argument("--seed", type=int, default=1)
     ap.add_argument("--mode", default="pgc", choices=["pgc", "is_sgd", "gc", "naive_cr"],
                     help="training scheme on the same kernels: PGC, or the IS-SGD / GC (FR) baselines")
@@ -60,7 +66,7 @@ def parse_args(argv=None):
 
 
 def workload_from_args(args) -> W.Workload:
-    w = W.WORKLOADS[args.workload]
+    w = W.WORKLOADS[args.workload or HEADLINE_WORKLOAD]
     kw = {}
     for o in args.override:
         k, v = o.split("=", 1)
@@ -351,8 +357,12 @@ def time_oracle(w: W.Workload, Xs, ys, masks, budget_s: float, min_steps: int = 
 
 
 # ---------------------------------------------------------------------------
-# distributed helpers (independent replicas; only timing is reduced)
+# one GPU only
 # ---------------------------------------------------------------------------
+
+SINGLE_GPU_ONLY = ("this path simulates all n workers of a PGC step on one GPU and has no multi-GPU form; "
+                   "run bench.py with --gpus 1 (no torchrun)")
+
 
 def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -361,58 +371,48 @@ def dist_env():
     return world, rank, local
 
 
-def max_over_ranks(value: float, world: int, device=None) -> float:
-    if world <= 1:
-        return value
-    import torch
-    import torch.distributed as dist
-    t = torch.tensor([value], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
-
-
-def job_value(ms_per_step_max: float, world: int) -> float:
-    """Whole-job steps/s: every replica runs its own copy of the workload
-    (weak scaling), so the job completes `world` steps per slowest-rank step."""
-    return world * 1000.0 / ms_per_step_max
-
-
-def barrier(world: int):
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
+def refuse_multi_gpu(args) -> None:
+    """The GPU arm runs on one GPU: with --gpus > 1, or under a launcher that
+    started several ranks, it stops here, before torch or the library is
+    imported, so no rank makes a CUDA call."""
+    world, _, _ = dist_env()
+    if args.gpus != 1 or world != 1:
+        print(json.dumps({"error": SINGLE_GPU_ONLY, "gpus": args.gpus, "world_size": world}), file=sys.stderr,
+              flush=True)
+        raise SystemExit(2)
 
 
 # ---------------------------------------------------------------------------
-# arms
+# the GPU arm
 # ---------------------------------------------------------------------------
 
 def default_steps(w: W.Workload) -> int:
+    """Steps of about two seconds of streaming work (20 to 20,000)."""
     per_step_bytes = evaluated_rows(w) * grad_bytes_per_row(w)
     est_s = max(per_step_bytes / 5.0e12, 20e-6)
+    if tensor_core_path(w):
+        est_s = max(est_s, 4.0 * evaluated_rows(w) * w.d * w.K / 1.2e15)
     return int(min(20000, max(20, 2.0 / est_s)))
 
 
-def run_ours(args):
-    import torch
-    world, rank, local = dist_env()
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
+def measure(w: W.Workload, K_steps: int, Wu: int, seed: int, mode: str, cpu_seconds, one_thread_seconds,
+            torch, dev) -> dict:
+    """Every measured field of one workload: device-timed steps/s, the
+    per-kernel-group breakdown, the dominant kernel's roofline, the end-to-end
+    rate through the public API with host buffers, the clocks during the
+    timed region, the simulated wall clock and (cpu_seconds not None) the
+    oracle on the host cores."""
     from paper_2607_20739_gb300 import binding as B
 
-    w = workload_from_args(args)
-    K_steps = args.steps or default_steps(w)
-    Wu = max(3, args.warmup)
-    Xs, ys = W.make_partitions(w, args.seed)
-    masks = W.make_masks(w, K_steps + Wu + 1, args.seed + 1000)
+    t_gen = time.perf_counter()
+    Xs, ys = W.make_partitions(w, seed)
+    masks = W.make_masks(w, K_steps + Wu + 1, seed + 1000)
+    gen_s = time.perf_counter() - t_gen
 
     stream = torch.cuda.Stream(device=dev)
-    g = B.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream, mode=args.mode)
+    g = B.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr, stream=stream, mode=mode)
     g.load(Xs, ys)
-    if args.mode == "naive_cr" or (args.mode == "gc" and w.scheme == "CR"):
+    if mode == "naive_cr" or (mode == "gc" and w.scheme == "CR"):
         g.set_gc_encoding(W.make_gc_draws(w, GC_DRAWS_SEED))
     P = w.K * w.d
     gout = torch.empty(P, device=dev)
@@ -432,10 +432,10 @@ def run_ours(args):
         do_step(t)
     g.sync()
 
-    # ---- device-timed region (no per-kernel events: they would break the
-    # programmatic-dependent overlap between consecutive step kernels) ------
-    clk = ClockSampler(local)
-    barrier(world)
+    # ---- device-timed region: exactly K_steps steps on the library's stream
+    # (no per-kernel events: they would break the programmatic-dependent
+    # overlap between consecutive step kernels) -----------------------------
+    clk = ClockSampler(int(dev.index or 0))
     torch.cuda.synchronize(dev)
     clk.start()
     time.sleep(0.25)
@@ -449,7 +449,6 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     region_ms = ev0.elapsed_time(ev1)
     clocks = clk.stop()
-    barrier(world)
 
     # ---- per-kernel-group breakdown: a second pass with events around each
     # group of every step, on the library's stream --------------------------
@@ -460,48 +459,55 @@ def run_ours(args):
     tim = g.timing_read()
     g.timing(False)
     launches_per_step = sum(tim["launches"]) / max(1, tim["steps"])
+    nsteps = max(1, tim["steps"])
+    group_ms = [m / nsteps for m in tim["ms"]]
     if flush:
-        ms_per_step = sum(tim["ms"]) / max(1, tim["steps"])
+        # the flush between steps is excluded: the step is its kernel groups
+        ms_per_step = sum(group_ms)
     else:
         ms_per_step = region_ms / K_steps
-    ms_per_step = max_over_ranks(ms_per_step, world, dev)
-    value = job_value(ms_per_step, world)
+    value = 1000.0 / ms_per_step
 
     # ---- roofline of the dominant kernel (streaming paths: the gradient
     # kernel, whose launch is the whole step when it carries the fused tail;
     # tensor-core softmax: the slower of the two GEMMs) ----------------------
     peaks, peak_src = load_peaks()
     bound, units, unit, peak = roofline_model(w, peaks)
-    nsteps = max(1, tim["steps"])
-    group_ms = [m / nsteps for m in tim["ms"]]
     single = all(n == 0 for n in tim["launches"][1:]) and tim["launches"][0] == tim["steps"]
     dom = 0
     if tensor_core_path(w) and group_ms[2] > group_ms[0]:
         dom = 2
     grad_ms = ms_per_step if (single and not flush) else group_ms[dom]
-    if unit == "GB/s":
-        achieved = units / (grad_ms * 1e-3) / 1e9
-    else:
-        achieved = units / (grad_ms * 1e-3) / 1e12
-    traffic = recorded_traffic(w.name)
+    scale = 1e9 if unit == "GB/s" else 1e12
+    achieved = units / (grad_ms * 1e-3) / scale
+    roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                "peak_source": peak_src, "kernel": kernel_label(w, single, dom), "duration_ms": grad_ms,
+                "traffic": recorded_traffic(w.name), "algorithmic_per_launch": units}
+    if tensor_core_path(w):
+        # the whole step against the burst rate: both contractions' flops
+        step_flops = 2.0 * units
+        burst = peaks.get("bf16_tflops") or 1900.0
+        roofline["step"] = {"flops": step_flops, "achieved": step_flops / (ms_per_step * 1e-3) / 1e12,
+                            "peak": burst, "unit": "TFLOP/s",
+                            "frac": step_flops / (ms_per_step * 1e-3) / 1e12 / burst,
+                            "note": "logits X W^T and gradient R^T X, 2 rows d K flops each, over the whole "
+                                    "step (both GEMMs, the commit into the stores and the decode) against the "
+                                    "burst bf16 rate"}
 
     # ---- end to end through the public API with host buffers -------------
-    g2 = g
     gh = torch.empty(P, dtype=torch.float32).pin_memory()
     wh = torch.empty(P, dtype=torch.float32).pin_memory()
     e2e_steps = max(10, min(K_steps, 2000))
-    barrier(world)
     t0 = time.perf_counter()
     for t in range(e2e_steps):
-        g2.step(mptr[t % len(mptr)], gh, wh, info=False)
+        g.step(mptr[t % len(mptr)], gh, wh, info=False)
     e2e_s = time.perf_counter() - t0
-    e2e_s = max_over_ranks(e2e_s, world, dev)
-    e2e_value = world * e2e_steps / e2e_s
+    e2e_value = e2e_steps / e2e_s
 
     # ---- the GC-CR modes' decoding coefficients alpha_{m,k} (§V-A): their
     # range, read after each of some untimed steps ------------------------
     alpha = None
-    if args.mode == "naive_cr" or (args.mode == "gc" and w.scheme == "CR"):
+    if mode == "naive_cr" or (mode == "gc" and w.scheme == "CR"):
         amax, amin, big = -float("inf"), float("inf"), 0
         na = min(200, len(mptr))
         for t in range(na):
@@ -511,42 +517,46 @@ def run_ours(args):
             big += int(max(abs(hi), abs(lo)) > 100.0)
         alpha = {"max": amax, "min": amin, "steps": na, "steps_with_abs_over_100": big,
                  "note": "alpha_{m,k} = d_m(J) c_{j_m,l} derived on the device each step (untimed steps)"}
+    g.close()
+    del gout, wout, flush_buf, gh, wh
+    torch.cuda.empty_cache()
 
-    # ---- cpu baseline (rank 0, N = 1 only) -------------------------------
+    # ---- cpu baseline: the oracle as it stands, on the host cores ---------
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, k, el, desc = time_oracle(w, Xs, ys, masks, args.cpu_seconds, mode=args.mode)
+    if cpu_seconds is not None:
+        v, k, el, desc = time_oracle(w, Xs, ys, masks, cpu_seconds, mode=mode)
         cpu = {"value": v, "unit": "steps/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": desc + "; fp64 numpy, BLAS threads = all cores", "cpu_model": cpu_model()}
-        if w.name in ONE_THREAD_WORKLOADS:
-            one = time_oracle_one_thread(w, args.seed, args.mode, min(8.0, args.cpu_seconds))
+        if w.name in ONE_THREAD_WORKLOADS and one_thread_seconds:
+            one = time_oracle_one_thread(w, seed, mode, one_thread_seconds)
             if one is not None:
                 cpu["value_1thread"] = one[0]
                 cpu["sample_1thread"] = one[1] + "; fp64 numpy, one thread"
-    g.close()
+    del Xs, ys
 
     # ---- simulated wall clock of a step (the paper's time per step, PGC vs
-    # DGD / IS-SGD / GC): measured compute and decode, seeded delays in units
-    # of the compute time --------------------------------------------------
+    # DGD / IS-SGD / GC): the device-timed step less the decode is the
+    # workers' compute, the decode is the master's; seeded delays in units of
+    # the compute time ------------------------------------------------------
     from paper_2607_20739_gb300 import wallclock as WC
-    # one partition per worker: a GC run measures c partitions per worker
-    compute_s = sum(group_ms[:3]) * 1e-3 / (w.c if args.mode == "gc" else 1)
-    decode_s = sum(group_ms[3:]) * 1e-3
-    delays = W.draw_delays(w, K_steps + Wu + 1, args.seed + 1000)[Wu:Wu + K_steps]
-    sim = WC.summary(delays, w.n, w.s, compute_s, compute_s, decode_s)
+    decode_ms = min(group_ms[4], ms_per_step)
+    compute_ms = ms_per_step - decode_ms
+    # one partition per worker: a GC run evaluates c partitions per worker
+    compute_s = compute_ms * 1e-3 / (w.c if mode == "gc" else 1)
+    delays = W.draw_delays(w, K_steps + Wu + 1, seed + 1000)[Wu:Wu + K_steps]
+    sim = WC.summary(delays, w.n, w.s, compute_s, compute_s, decode_ms * 1e-3)
     sim["model"] = ("each worker finishes after (partitions evaluated) x compute + delay; the master waits for "
                     "the n - s fastest (pgc, is_sgd, gc with c partitions per worker) or all n (dgd), then decodes; "
-                    "delays are the seeded draws that pick the stragglers, in units of the compute time")
+                    "compute = the device-timed step less its decode kernel (per partition), decode = the decode "
+                    "kernel's event time; delays are the seeded draws that pick the stragglers, in units of the "
+                    "compute time")
 
     uniq = evaluated_rows(w)
-    line = {
-        "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": K_steps, "warmup": Wu,
-        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+    out = {
+        "value": value, "unit": "steps/s", "steps": K_steps, "warmup": Wu, "ms_per_step": ms_per_step,
         "dtype": "f32" if w.dtype == "f32" else "bf16-in/f32-acc",
-        "data": f"synthetic, seeded (seed {args.seed}); {w.features} features, planted-model labels, "
-                f"{w.delays} straggler delays",
         "config": {"workload": w.name, "scheme": w.scheme, "n": w.n, "s": w.s, "loss": w.loss, "d": w.d, "K": w.K,
-                   "rows_per_partition": w.m, "features": w.dtype, "parallelism": f"replicas{world}", "mode": args.mode,
+                   "rows_per_partition": w.m, "features": w.dtype, "parallelism": "single GPU", "mode": mode,
                    "l2": ("flushed between steps (256 MiB write, excluded from step time)" if flush else
                           f"inputs larger than L2: {step_bytes / 2**20:.0f} MiB streamed per step")},
         "samples_per_s_unique": value * uniq,
@@ -555,27 +565,68 @@ def run_ours(args):
                                if tim["launches"][i] > 0},
         "kernel_timing_note": "per-group CUDA events from a separate pass; events between launches "
                               "serialise the dependent-launch overlap, so these sum to more than ms_per_step",
-        "roofline": {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
-                     "peak_source": peak_src, "kernel": kernel_label(w, single, dom),
-                     "duration_ms": grad_ms, "traffic": traffic,
-                     "algorithmic_per_launch": units},
+        "roofline": roofline,
         "cpu_baseline": cpu,
-        "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": w.n,
+        "e2e": {"value": e2e_value, "unit": "steps/s", "steps": e2e_steps, "h2d_bytes_per_step": w.n,
                 "d2h_bytes_per_step": 2 * P * 4},
         "gpu_launches": int(round(launches_per_step * K_steps)),
         "simulated_wall_clock": sim,
         "clocks": clocks,
+        "input_generation_s": gen_s,
     }
     if alpha is not None:
-        line["decoding_coefficients"] = alpha
-    if rank == 0:
-        print(json.dumps(line), flush=True)
-    if world > 1:
-        import torch.distributed as dist
-        dist.destroy_process_group()
+        out["decoding_coefficients"] = alpha
+    return out
+
+
+def run_ours(args):
+    refuse_multi_gpu(args)
+    import torch
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py: no CUDA device (the GPU arm has no CPU fallback)")
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
+
+    head = workload_from_args(args)
+    K_steps = args.steps or default_steps(head)
+    Wu = max(3, args.warmup)
+    cpu_s = None if args.no_cpu_baseline else args.cpu_seconds
+    res = measure(head, K_steps, Wu, args.seed, args.mode, cpu_s, min(8.0, args.cpu_seconds), torch, dev)
+
+    per = None
+    if args.workload is None and not args.no_per_workload:
+        # every other workload in the same invocation, each over its own
+        # step count (about two seconds of work) with 5 warm-up steps
+        per = {}
+        cpu_o = None if args.no_cpu_baseline else min(args.cpu_seconds, 8.0)
+        for name in W.WORKLOAD_ORDER:
+            if name == head.name:
+                continue
+            w = W.WORKLOADS[name]
+            per[name] = measure(w, default_steps(w), 5, args.seed, args.mode, cpu_o, min(5.0, args.cpu_seconds),
+                                torch, dev)
+
+    line = {
+        "metric": METRIC, "value": res["value"], "unit": "steps/s", "n_gpus": 1, "steps": K_steps, "warmup": Wu,
+        "ms_per_step": res["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": res["dtype"],
+        "data": f"synthetic, seeded (seed {args.seed}); {head.features} features, planted-model labels, "
+                f"{head.delays} straggler delays",
+    }
+    for k, v in res.items():
+        if k not in line:
+            line[k] = v
+    if per is not None:
+        line["per_workload"] = per
+        line["per_workload_note"] = ("the other workloads, measured in this invocation after the headline, each "
+                                     "over its own step count (about two seconds of device work) after 5 warm-up "
+                                     "steps; every field as at the top level")
+    print(json.dumps(line), flush=True)
 
 
 def run_reference(args):
+    """The fp64 oracle on the host cores (CPU only: no CUDA call).  Under a
+    launcher that started several ranks only rank 0 runs it."""
     world, rank, _ = dist_env()
     if rank != 0:
         return

@@ -355,7 +355,10 @@ int pgc_timing_read(pgc_ctx *ctx, double *ms, int64_t *launches, int64_t *steps_
  * Scratch: a fixed 16 MiB array inside the library (a __device__ global),
  * held on every GPU that loads the library until the process exits.  The
  * first call on a device looks up the array's device address (with that
- * device current); make that first call before any stream capture.  All
+ * device current) and keeps it for the life of the process; make that first
+ * call before any stream capture.  cudaDeviceReset on a device unloads the
+ * library's module there and makes the kept address stale: a process that
+ * resets a device must not call this entry point on it afterwards.  All
  * calls share the array and it keeps the last call's contents; each call
  * rewrites what it reads, but calls that overlap on the GPU (other streams,
  * other threads) race on it.

@@ -14,7 +14,9 @@
 // exits.  Host code cannot use the array's name as a device address, so the
 // first call on each device, with that device current, looks the address up
 // with cudaGetSymbolAddress and caches it; that first call should therefore
-// come before any stream capture.  The call then fills its small work tables
+// come before any stream capture.  The cached address is not refreshed: after
+// cudaDeviceReset (which unloads this module on that device) it is stale, so
+// a process that resets a device must not call this entry point there again.  The call then fills its small work tables
 // in the scratch with a kernel, runs the streaming gradient kernel (partial
 // sums per CTA into the scratch) and the commit kernel (ordered sum of those
 // partials, scaled by 1/m, into the caller's output), waits for the stream

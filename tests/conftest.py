@@ -13,6 +13,23 @@ def pytest_configure(config):
     config.addinivalue_line("markers", "slow: long-running")
 
 
+_HEADROOM: list[str] = []
+
+
+@pytest.fixture(scope="session")
+def headroom():
+    """Lines "case: worst observed error against its tolerance", printed after
+    the run, so the margin of every floating-point parity check is on record."""
+    return _HEADROOM
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    if _HEADROOM:
+        terminalreporter.section("parity headroom: worst observed error / tolerance")
+        for line in _HEADROOM:
+            terminalreporter.write_line(line)
+
+
 @pytest.fixture(scope="session")
 def root_dir():
     return ROOT

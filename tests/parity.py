@@ -70,25 +70,35 @@ def run_gpu(binding, w: W.Workload, Xs, ys, masks, record_loss=True, mode="pgc")
     return g, out
 
 
-def compare_runs(w: W.Workload, gpu_recs, ora_recs, check_loss=True):
+def compare_step(w: W.Workload, t: int, a: dict, b: dict, check_loss=True):
+    """One step of a GPU record `a` against the oracle's `b`: schedule, slot,
+    FR representatives and the decode support bit-exact, the coefficients to
+    fp32 rounding, the decoded gradient within GRAD_TOL and (check_loss) the
+    loss F(beta^(t)) within LOSS_TOL.  Returns (gradient error, loss error)."""
     tol = GRAD_TOL[w.dtype]
+    assert a["t"] == b["t"] == t
+    assert a["slot"] == b["slot"], (t, a["slot"], b["slot"])
+    assert list(a["eval_partition"]) == list(b["eval_partition"]), t
+    if w.scheme == "FR":
+        assert list(a["fr_rep"]) == list(b["fr_rep"]), t
+    assert a["received"] == b["received"]
+    # device-derived coefficients: same support, same values (fp32)
+    ca = np.asarray(a["coeff"], dtype=np.float64)
+    cb = np.asarray(b["coeff"], dtype=np.float64)
+    assert ((ca != 0) == (cb != 0)).all(), (t, ca, cb)
+    np.testing.assert_allclose(ca, cb, rtol=2e-7, atol=0)
+    e = rel_err(a["grad"], b["grad"])
+    assert e <= tol, f"step {t}: decoded-gradient error {e:.3g} > {tol}"
+    le = 0.0
+    if check_loss and a["loss"] is not None:
+        le = abs(a["loss"] - b["loss"]) / abs(b["loss"])
+        assert le <= LOSS_TOL, f"step {t}: loss {a['loss']} vs {b['loss']} ({le:.3g})"
+    return e, le
+
+
+def compare_runs(w: W.Workload, gpu_recs, ora_recs, check_loss=True):
     worst = 0.0
     for t, (a, b) in enumerate(zip(gpu_recs, ora_recs)):
-        assert a["t"] == b["t"] == t
-        assert a["slot"] == b["slot"], (t, a["slot"], b["slot"])
-        assert list(a["eval_partition"]) == list(b["eval_partition"]), t
-        if w.scheme == "FR":
-            assert list(a["fr_rep"]) == list(b["fr_rep"]), t
-        assert a["received"] == b["received"]
-        # device-derived coefficients: same support, same values (fp32)
-        ca = np.asarray(a["coeff"], dtype=np.float64)
-        cb = np.asarray(b["coeff"], dtype=np.float64)
-        assert ((ca != 0) == (cb != 0)).all(), (t, ca, cb)
-        np.testing.assert_allclose(ca, cb, rtol=2e-7, atol=0)
-        e = rel_err(a["grad"], b["grad"])
+        e, _ = compare_step(w, t, a, b, check_loss)
         worst = max(worst, e)
-        assert e <= tol, f"step {t}: decoded-gradient error {e:.3g} > {tol}"
-        if check_loss and a["loss"] is not None:
-            le = abs(a["loss"] - b["loss"]) / abs(b["loss"])
-            assert le <= LOSS_TOL, f"step {t}: loss {a['loss']} vs {b['loss']} ({le:.3g})"
     return worst
