@@ -463,7 +463,8 @@ def measure(w: W.Workload, K_steps: int, Wu: int, seed: int, mode: str, cpu_seco
     group_ms = [m / nsteps for m in tim["ms"]]
     if flush:
         # the flush between steps is excluded: the step is its kernel groups
-        ms_per_step = sum(group_ms)
+        # (groups that launched nothing hold only the events' own time)
+        ms_per_step = sum(m for m, nl in zip(group_ms, tim["launches"]) if nl > 0)
     else:
         ms_per_step = region_ms / K_steps
     value = 1000.0 / ms_per_step

@@ -17,14 +17,19 @@
 //      16 x 16 block to the other CTA with st.async into distributed shared
 //      memory, add the two blocks in rank order (so both CTAs form the same
 //      R) and form R = softmax(Z) - onehot(y) (zero past K and past the
-//      partition's rows) in bf16, in the no-swizzle K-major operand layout;
+//      partition's rows) as two bf16 blocks, R_hi = bf16(R) and R_lo =
+//      bf16(R - R_hi), in the no-swizzle K-major operand layout (R alone in
+//      bf16 is not enough: when the rows' softmax values are alike, their
+//      rounding errors are alike too and add up coherently over the rows of
+//      the contraction with non-negative features);
 //   3. the same eight warps copy the half tile, transposed, into tensor memory
 //      (one lane per feature, two rows per 32-bit column: the K-major A
 //      operand of the gradient MMA) and release the slot, so a slot is held
 //      only for its load, the logits and the copy, not for the exchange of
 //      step 2; kNA copies (and R blocks) rotate;
 //   4. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
-//      the 16 rows; A = the tile's copy in tensor memory, B = R) into a TMEM
+//      the 16 rows; A = the tile's copy in tensor memory, B = R_hi, then
+//      again with B = R_lo) into a TMEM
 //      accumulator of the CTA's half of G^T that spans the pair's run of tiles
 //      in a partition; its commit frees the copy and the R block.
 // No data leaves the pair before the end of a run; then the eight warps write
@@ -57,7 +62,7 @@ constexpr int kRThreads = 64 + 32 * kFw + 32 * kNRes;
 // 16-feature steps per forward warp at the largest ld
 constexpr int kMaxKs = (int)(kRowsMaxLd / kPairCtas / (16 * kFw));
 constexpr uint32_t kZp = kRR * 16 * 4;   // a 16 x 16 fp32 block of partial logits
-constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16)
+constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16); R_lo blocks follow the kNA R_hi
 constexpr int kNA = 3;                   // tiles whose gradient MMA may be pending (TMEM copies, R blocks)
 constexpr int kTmemCols = 512;           // G^T half, then the kNA copies of a tile
 constexpr uint32_t kAccCols = 192;       // G^T half: ld / 256 slices of 16 columns at the largest ld
@@ -203,7 +208,8 @@ __device__ bool grid_barrier(int* ctr, int* status, int* flag) {
 
 // Shared memory of a CTA: slots of its half tile, two sets (tile parity) of
 // the forward warps' partial logits (the fused tail's decode plan reuses
-// them), two blocks for the other CTA's partial, kNA R blocks, barriers.
+// them), two blocks for the other CTA's partial, kNA R_hi then kNA R_lo
+// blocks, barriers.
 struct RowsSmem {
   uint32_t slot_bytes, zpart, zpeer, rblk, bars, total;
 };
@@ -214,7 +220,7 @@ __host__ __device__ static RowsSmem rows_smem(int64_t ld, int nslots) {
   s.zpart = (uint32_t)nslots * s.slot_bytes;
   s.zpeer = s.zpart + 2 * kFw * kZp;
   s.rblk = s.zpeer + 2 * kZp;
-  s.bars = s.rblk + (uint32_t)kNA * kRb;
+  s.bars = s.rblk + 2u * (uint32_t)kNA * kRb;
   s.total = s.bars + kRowsBars * 8 + 16;
   return s;
 }
@@ -329,13 +335,17 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       if (first && run > 0 && !mbar_wait(acc_empty, (run - 1) & 1, a.status)) { ok = false; break; }
       tc_fence_after();
       const uint64_t db = sdesc(smem_u32(rblk + ab * kRb), 256, 128, 0);
+      const uint64_t dbl = sdesc(smem_u32(rblk + (kNA + ab) * kRb), 256, 128, 0);
       // slice mt: its 128 features x 16 rows are columns kAccCols + ab kAStride + 8 mt ..
       const uint32_t ta = tmem + kAccCols + (uint32_t)ab * kAStride;
-      if (first) {
-        for (int mt = 0; mt < nmt; ++mt) umma_ta_fresh(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), db, id_bwd);
-      } else {
-        for (int mt = 0; mt < nmt; ++mt) umma_ta_acc(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), db, id_bwd);
+      // all slices with R_hi, then all with R_lo: consecutive MMAs write
+      // different accumulators
+      for (int mt = 0; mt < nmt; ++mt) {
+        const uint32_t d = tmem + (uint32_t)(mt * 16), am = ta + (uint32_t)(mt * 8);
+        if (first) umma_ta_fresh(d, am, db, id_bwd);
+        else umma_ta_acc(d, am, db, id_bwd);
       }
+      for (int mt = 0; mt < nmt; ++mt) umma_ta_acc(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), dbl, id_bwd);
       umma_commit(&a_empty[ab]);
       if (last) {
         umma_commit(acc_full);
@@ -419,11 +429,15 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         break;
       }
       uint8_t* blk = rblk + (i % kNA) * kRb;
+      uint8_t* blk_lo = rblk + (kNA + i % kNA) * kRb;
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         const int k = kh + c;
         const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
-        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, k_of_row(r))) = __float2bfloat16_rn(v);
+        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+        const uint32_t off = r_offset(k, k_of_row(r));
+        *reinterpret_cast<__nv_bfloat16*>(blk + off) = hi;
+        *reinterpret_cast<__nv_bfloat16*>(blk_lo + off) = __float2bfloat16_rn(v - __bfloat162float(hi));
       }
       fence_proxy_async_smem();
       __syncwarp();

@@ -12,11 +12,14 @@
 //      M = 128 rows, N = 16 classes, accumulator in TMEM);
 //   2. the partial Z rows are sent to their owner CTA (rank = row / 16) with
 //      st.async into distributed shared memory; the owner sums the 8 slices,
-//      forms R = softmax(Z) - onehot(y) for its 16 rows and sends that bf16
-//      block to all 8 CTAs with bulk copies (cp.async.bulk shared::cluster);
+//      forms R = softmax(Z) - onehot(y) for its 16 rows and sends it to all 8
+//      CTAs with bulk copies (cp.async.bulk shared::cluster) as two bf16
+//      blocks, R_hi = bf16(R) and R_lo = bf16(R - R_hi): bf16 alone is not
+//      enough when the rows' softmax values are alike, since their rounding
+//      errors then add up coherently over the rows of the contraction;
 //   3. each CTA accumulates its slice of G^T (M = 128 features, N = 16
-//      classes, K = the tile's rows) in TMEM, reading the same resident X
-//      slice, now as an MN-major operand.
+//      classes, K = the tile's rows; B = R_hi, then B = R_lo) in TMEM,
+//      reading the same resident X slice, now as an MN-major operand.
 // When a cluster's run of tiles leaves a partition its G^T slices are written
 // as one partial (one item per cluster and partition); a separate commit
 // kernel sums the items of each partition, scales by 1/m_e and writes the
@@ -175,7 +178,7 @@ __device__ __forceinline__ uint32_t r_offset(int k, int r) {
 
 // Shared-memory plan; offsets from the 1024-byte aligned base.
 struct SkSmem {
-  uint32_t slots, slot_bytes, wsm, zred, rstage, rbuf, tiles, bars, total;
+  uint32_t slots, slot_bytes, wsm, zred, rstage, rbuf, rbuf_lo, tiles, bars, total;
 };
 __host__ __device__ static SkSmem sk_smem(int nper) {
   SkSmem s;
@@ -185,8 +188,9 @@ __host__ __device__ static SkSmem sk_smem(int nper) {
   s.wsm = 2 * s.slot_bytes;
   s.zred = s.wsm + (uint32_t)((nper * kWBox + 1023) & ~1023);
   s.rstage = s.zred + kCS * kZPart;
-  s.rbuf = s.rstage + 2 * kRBlock;
-  s.tiles = s.rbuf + 2 * kCS * kRBlock;
+  s.rbuf = s.rstage + 4 * kRBlock;          // staging: [slot][hi, lo]
+  s.rbuf_lo = s.rbuf + 2 * kCS * kRBlock;
+  s.tiles = s.rbuf_lo + 2 * kCS * kRBlock;
   s.bars = s.tiles + kTileCache * 16;
   s.total = s.bars + 32 * 8 + 16;
   return s;
@@ -202,6 +206,7 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
   float* zred = reinterpret_cast<float*>(sm + L.zred);
   uint8_t* rstage = sm + L.rstage;
   uint8_t* rbuf = sm + L.rbuf;
+  uint8_t* rbuf_lo = sm + L.rbuf_lo;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.bars);
   uint64_t* slot_full = bars + 0;    // [2]
   uint64_t* slot_empty = bars + 2;   // [2]
@@ -256,8 +261,8 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
   // the receive barriers expect their first tiles before any peer can send
   if (threadIdx.x == 64) {
     mbar_arrive_expect_tx(zred_full, kCS * kZPart);
-    mbar_arrive_expect_tx(&rfull[0], kCS * kRBlock);
-    mbar_arrive_expect_tx(&rfull[1], kCS * kRBlock);
+    mbar_arrive_expect_tx(&rfull[0], 2 * kCS * kRBlock);
+    mbar_arrive_expect_tx(&rfull[1], 2 * kCS * kRBlock);
   }
   fence_before();
   cl_sync();
@@ -320,16 +325,19 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
         const int g = (seg + (first ? 1 : 0)) & 1;
         if (!first || seg + 1 < 2 || mbar_test_wait(&gempty[g], (((seg + 1) >> 1) - 1) & 1)) {
           if (first) ++seg;
-          if (b + 2 < n) mbar_arrive_expect_tx(&rfull[s], kCS * kRBlock);
+          if (b + 2 < n) mbar_arrive_expect_tx(&rfull[s], 2 * kCS * kRBlock);
           fence_after();
           const uint32_t base = smem_u32(slot0 + s * L.slot_bytes);
           const uint64_t db = sdesc(smem_u32(rbuf + s * kCS * kRBlock), 256, 128, 0);
+          const uint64_t dbl = sdesc(smem_u32(rbuf_lo + s * kCS * kRBlock), 256, 128, 0);
           for (int mt = 0; mt < nmt; ++mt) {
             const uint64_t da = sdesc(base + 2 * mt * kBox, kBox, 1024, 2);
             const uint32_t d = tmem + gacc_col(g) + mt * kNC;
             mma(d, da, db, id_bwd, first ? 0u : 1u);
 #pragma unroll
             for (int kk = 1; kk < kRows / 16; ++kk) mma_acc(d, da + kk * 128, db + kk * 32, id_bwd);
+#pragma unroll
+            for (int kk = 0; kk < kRows / 16; ++kk) mma_acc(d, da + kk * 128, dbl + kk * 32, id_bwd);
           }
           commit(&slot_empty[s]);
           if (last) commit(&gfull[g]);
@@ -430,15 +438,24 @@ softmax_smallk_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_cons
       const float inv = 1.0f / sum;
       const float ra = valid && k0 < a.K ? ea * inv - (k0 == lab ? 1.f : 0.f) : 0.f;
       const float rb = valid && k1 < a.K ? eb * inv - (k1 == lab ? 1.f : 0.f) : 0.f;
-      uint8_t* blk = rstage + s * kRBlock;
-      *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k0, j)) = __float2bfloat16_rn(ra);
-      *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k1, j)) = __float2bfloat16_rn(rb);
+      uint8_t* blk = rstage + 2 * s * kRBlock;
+      uint8_t* blk_lo = blk + kRBlock;
+      {
+        const __nv_bfloat16 ha = __float2bfloat16_rn(ra), hb = __float2bfloat16_rn(rb);
+        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k0, j)) = ha;
+        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k1, j)) = hb;
+        *reinterpret_cast<__nv_bfloat16*>(blk_lo + r_offset(k0, j)) = __float2bfloat16_rn(ra - __bfloat162float(ha));
+        *reinterpret_cast<__nv_bfloat16*>(blk_lo + r_offset(k1, j)) = __float2bfloat16_rn(rb - __bfloat162float(hb));
+      }
       fence_proxy_async_smem();
       named_sync(1, 128);
       if (t == 0) {
         const uint32_t dst_off = smem_u32(rbuf + s * kCS * kRBlock) + rank * kRBlock;
-        for (uint32_t d = 0; d < (uint32_t)kCS; ++d)
+        const uint32_t dst_lo = smem_u32(rbuf_lo + s * kCS * kRBlock) + rank * kRBlock;
+        for (uint32_t d = 0; d < (uint32_t)kCS; ++d) {
           bulk_s2cluster(mapa(dst_off, d), blk, kRBlock, mapa(smem_u32(&rfull[s]), d));
+          bulk_s2cluster(mapa(dst_lo, d), blk_lo, kRBlock, mapa(smem_u32(&rfull[s]), d));
+        }
       }
       // (4) end of this cluster's run in a partition: write the G^T slices
       if (last) {

@@ -23,6 +23,8 @@ CASES = {
     "cr_logistic": ("pgc", WL["cr_n8_logistic_d1024"].replace(m=300, d=200), 7, 3, True),
     "fr_softmax_smallk": ("pgc", WL["fr_n32_softmax_k10"].replace(n=8, m=150), 6, 2, True),
     "cr_softmax_tensor_core": ("pgc", WL["cr_n128_softmax_k1000"].replace(n=5, s=2, K=300, d=320, m=130), 6, 4, False),
+    # P = K d >= 2^20: the one-thread-per-column decode
+    "cr_softmax_wide_decode": ("pgc", WL["cr_n128_softmax_k1000"].replace(n=5, s=2, K=256, d=4096, m=64), 7, 3, False),
     "is_sgd_lsq": ("is_sgd", WL["cr_n64_lsq_d16384"].replace(n=6, s=2, d=700, m=40), 5, 2, True),
 }
 
@@ -70,7 +72,9 @@ def test_resume_follows_the_oracle(libpgc, cuda, headroom, name):
             np.testing.assert_array_equal(r1["grad"], r2["grad"])
             np.testing.assert_array_equal(r1["beta"], r2["beta"])
         else:
-            assert rel_err(r1["grad"], r2["grad"]) < 1e-5 and rel_err(r1["beta"], r2["beta"]) < 1e-6
+            # the slot total's reduce-adds land in completion order; a few
+            # free-running steps carry that rounding through the bf16 copy of beta
+            assert rel_err(r1["grad"], r2["grad"]) < 1e-5 and rel_err(r1["beta"], r2["beta"]) < 1e-5
 
 
 def test_checkpoint_of_another_configuration_is_refused(libpgc, cuda):

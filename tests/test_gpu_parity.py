@@ -65,14 +65,22 @@ def test_parity_with_oracle(libpgc, cuda, name):
     g.close()
 
 
-@pytest.mark.parametrize("name", ["fr_smallk_k10_unequal_rows", "cr_smallk_k16_d1000"])
+CLUSTER_CASES = {
+    "fr_smallk_k10_d2048_unequal_rows": (WL["fr_n32_softmax_k10"].replace(n=4, s=1, d=2048, m=(300, 1, 129, 700)), 5),
+    "cr_smallk_k16_d1000": CASES["cr_smallk_k16_d1000"],
+}
+
+
+@pytest.mark.parametrize("name", list(CLUSTER_CASES))
 def test_parity_cluster_few_class_kernel(libpgc, cuda, monkeypatch, name):
-    """The few-class cases again with the 8-CTA cluster kernel (the path taken
-    when the whole-row kernel does not apply)."""
+    """Few-class cases with the 8-CTA cluster kernel (the fall-back taken when
+    the whole-row kernel does not apply; its shared memory holds rows of up
+    to 2048 features)."""
     monkeypatch.setenv("PGC_NO_ROWS", "1")
-    w, T = CASES[name]
+    w, T = CLUSTER_CASES[name]
     Xs, ys, masks = generate(w, T)
     g, grecs = run_gpu(libpgc, w, Xs, ys, masks)
+    assert g.gradient_path == "softmax_cluster"
     orecs = run_oracle(w, Xs, ys, masks)
     compare_runs(w, grecs, orecs)
     g.close()
@@ -216,10 +224,15 @@ def test_gradient_path_chosen(libpgc, cuda, name):
 
 
 def test_gradient_path_overrides(libpgc, cuda, monkeypatch):
-    w, _ = CASES["fr_smallk_k10_unequal_rows"]
     monkeypatch.setenv("PGC_NO_ROWS", "1")
+    w, _ = CLUSTER_CASES["fr_smallk_k10_d2048_unequal_rows"]
     g = libpgc.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr)
     assert g.gradient_path == "softmax_cluster"
+    g.close()
+    # rows longer than the cluster kernel's shared memory holds: CUDA cores
+    w, _ = CASES["fr_smallk_k10_unequal_rows"]
+    g = libpgc.PGC(w.scheme, w.n, w.s, w.loss, w.dtype, w.d, K=w.K, rows=w.rows(), lr=w.lr)
+    assert g.gradient_path == "softmax_cc"
     g.close()
     w, _ = CASES["cr_tc_k300_d320_m200"]
     monkeypatch.setenv("PGC_NO_FUSED", "1")
