@@ -22,9 +22,18 @@
 // reduce-add per block at the end of the run.  So U costs one reduce per run
 // instead of one per partition.
 // Every wait is bounded; the TMEM allocation is released on every path.
+//
+// Pair form (kPair, the default): the same units and epilogue, but the
+// pair's MMA is one tcgen05.mma.cta_group::2 (M = 256 classes: 128 from each
+// CTA's TMEM and shared memory; N = 256 features: each CTA holds 128 of them)
+// issued by the even CTA.  A stage then holds 16 KB of R and 16 KB of X per
+// CTA instead of 16 + 32, so six stages fit where four did; each CTA's TMA
+// loads complete on the even CTA's stage barrier, and the MMA's commits free
+// the stage and hand over the accumulator in both CTAs.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
 #include <cstring>
 
 #include "tc_common.cuh"
@@ -34,9 +43,13 @@ namespace pgc {
 namespace {
 
 constexpr int kGM = 128, kGN = 256, kGK = 64;
-constexpr int kGS = 4;                          // shared-memory stages
 constexpr uint32_t kGA = kGM * kGK * 2;         // 16 KB R tile (two 64 x 64 boxes)
-constexpr uint32_t kGB = kGN * kGK * 2;         // 32 KB X tile (four 64 x 64 boxes)
+// per CTA: stages, and the X tile it holds (all 256 features, multicast
+// halves; or, in the pair form, its 128 of them)
+template <bool kPair> struct GradCfg {
+  static constexpr int kStages = kPair ? 6 : 4;
+  static constexpr uint32_t kB = (kPair ? kGN / 2 : kGN) * kGK * 2;   // 16 or 32 KB
+};
 constexpr int kGThreads = 320;                  // producer, MMA, 8 epilogue warps
 constexpr int kGEpi = 8;
 constexpr uint32_t kGTmem = 2 * kGN;            // two fp32 accumulators
@@ -45,9 +58,11 @@ constexpr uint32_t kGBox = 32 * 32 * 4;         // one 32 x 32 fp32 output box
 struct GradSmem {
   uint32_t sA, sB, box, bars, total;
 };
+template <bool kPair>
 __host__ __device__ constexpr GradSmem grad_smem() {
-  return GradSmem{0, kGS * kGA, kGS * (kGA + kGB), kGS * (kGA + kGB) + kGEpi * kGBox,
-                  kGS * (kGA + kGB) + kGEpi * kGBox + 16 * 8};
+  constexpr int S = GradCfg<kPair>::kStages;
+  constexpr uint32_t B = GradCfg<kPair>::kB;
+  return GradSmem{0, S * kGA, S * (kGA + B), S * (kGA + B) + kGEpi * kGBox, S * (kGA + B) + kGEpi * kGBox + 24 * 8};
 }
 
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
@@ -65,42 +80,56 @@ __device__ __forceinline__ void stage_quarter(uint8_t* box, int lane, int qt, co
 // Ten warps put three on some of the SM's four register-file quarters, so a
 // thread gets at most 168 registers; the epilogue keeps 128 partial sums of
 // the slot total in them and reads TMEM 16 columns at a time.
+template <bool kPair>
 __global__ void __launch_bounds__(kGThreads, 1)
 tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ CUtensorMap tmX,
                const __grid_constant__ CUtensorMap tmU, const __grid_constant__ CUtensorMap tmS, TcGradParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  constexpr GradSmem L = grad_smem();
+  constexpr int kGS = GradCfg<kPair>::kStages;
+  constexpr uint32_t kGB = GradCfg<kPair>::kB;
+  constexpr GradSmem L = grad_smem<kPair>();
   uint8_t* sA = sm + L.sA;
   uint8_t* sB = sm + L.sB;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.bars);
-  uint64_t* full = bars;                // [4]
-  uint64_t* empty = bars + 4;           // [4]
-  uint64_t* acc_full = bars + 8;        // [2]
-  uint64_t* acc_empty = bars + 10;      // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
-  int* cta_err = reinterpret_cast<int*>(bars + 13);
+  uint64_t* full = bars;                // [kGS]
+  uint64_t* empty = bars + kGS;         // [kGS]
+  uint64_t* acc_full = bars + 2 * kGS;  // [2]
+  uint64_t* acc_empty = acc_full + 2;   // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 4);
+  int* cta_err = reinterpret_cast<int*>(acc_full + 5);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rank = (int)cluster_rank();
-  constexpr uint16_t kPair = 0x3;
+  constexpr uint16_t kBoth = 0x3;
+  // pair form: the even CTA issues the MMAs and owns the stage and
+  // accumulator barriers they wait on
+  const bool issuer = !kPair || rank == 0;
   if (threadIdx.x == 0) {
     *cta_err = 0;
     for (int s = 0; s < kGS; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 2);           // the MMAs of both CTAs read the stage
+      mbar_init(&empty[s], kPair ? 1 : 2);   // the pair MMA's commit, or the MMAs of both CTAs
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&acc_full[a], 1);
-      mbar_init(&acc_empty[a], kGEpi);
+      mbar_init(&acc_empty[a], kPair ? 2 * kGEpi : kGEpi);   // pair form: both CTAs' epilogues
     }
     fence_mbar_init();
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                 "r"(kGTmem)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if constexpr (kPair) {
+      // one warp of each CTA of the pair allocates, together
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                   "r"(kGTmem)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                   "r"(kGTmem)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   tc_fence_before();
   cluster_sync_all();                    // the peer's barriers exist before any multicast
@@ -125,25 +154,38 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const int s = it % kGS;
           if (it >= kGS && !mbar_wait(&empty[s], ((it / kGS) - 1) & 1, p.status)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[s], kGA + kGB);
           uint8_t* a_dst = sA + (size_t)s * kGA;
           uint8_t* b_dst = sB + (size_t)s * kGB;
-          for (int q = 0; q < 2; ++q)
-            tma_load_2d(a_dst + q * 8192, &tmR, mt * kGM + q * 64, p.a_off[b] + kb * kGK, &full[s]);
-          for (int q = 2 * rank; q < 2 * rank + 2; ++q)
-            tma_load_2d_mc(b_dst + q * 8192, &tmX, nt * kGN + q * 64, p.b_off[b] + kb * kGK, &full[s], kPair);
+          if constexpr (kPair) {
+            // this CTA's R rows and its 128 features of X, counted on the
+            // even CTA's stage barrier (which expects both CTAs' bytes)
+            if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * (kGA + kGB));
+            const uint32_t fb = cluster_addr(&full[s], 0);
+            for (int q = 0; q < 2; ++q)
+              tma_load_2d_pair(a_dst + q * 8192, &tmR, mt * kGM + q * 64, p.a_off[b] + kb * kGK, fb);
+            for (int q = 0; q < 2; ++q)
+              tma_load_2d_pair(b_dst + q * 8192, &tmX, nt * kGN + rank * 128 + q * 64, p.b_off[b] + kb * kGK, fb);
+          } else {
+            mbar_arrive_expect_tx(&full[s], kGA + kGB);
+            for (int q = 0; q < 2; ++q)
+              tma_load_2d(a_dst + q * 8192, &tmR, mt * kGM + q * 64, p.a_off[b] + kb * kGK, &full[s]);
+            for (int q = 2 * rank; q < 2 * rank + 2; ++q)
+              tma_load_2d_mc(b_dst + q * 8192, &tmX, nt * kGN + q * 64, p.b_off[b] + kb * kGK, &full[s], kBoth);
+          }
         }
       }
     }
     if (!ok) atomicExch(cta_err, 1);
     // no copy may outlive the CTA: wait for the last fill of every stage
+    // (pair form: the last MMA commit on a stage follows both CTAs' copies)
     for (int s = 0; s < kGS && s < it; ++s) {
       const int last = ((it - 1 - s) / kGS) * kGS + s;
-      mbar_wait(&full[s], (last / kGS) & 1, p.status);
+      if (kPair) mbar_wait(&empty[s], (last / kGS) & 1, p.status);
+      else mbar_wait(&full[s], (last / kGS) & 1, p.status);
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1 && lane == 0 && issuer) {
     // ---- MMA issuer --------------------------------------------------------
-    constexpr uint32_t idesc = idesc_bf16_f32(kGM, kGN, true, true);
+    constexpr uint32_t idesc = idesc_bf16_f32(kPair ? 2 * kGM : kGM, kGN, true, true);
     int it = 0, tt = 0;
     bool ok = true;
     for (int i = 0; i < my_units && ok; ++i) {
@@ -165,12 +207,17 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
             // MN-major: the next 16 K rows are two 8-row groups (2 KB) further
             const uint64_t da = smem_desc_sw128(a_base + kk * 2048, 8192, 1024);
             const uint64_t db = smem_desc_sw128(b_base + kk * 2048, 8192, 1024);
-            umma_bf16(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
+            if constexpr (kPair) umma_bf16_pair(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
+            else umma_bf16(d_tmem, da, db, idesc, (kb | kk) != 0 ? 1u : 0u);
           }
-          umma_commit_mc(&empty[s], kPair);  // this CTA is done with the stage, in both CTAs' count
+          // the stage is free again, in both CTAs
+          if constexpr (kPair) umma_commit_pair_mc(&empty[s], kBoth);
+          else umma_commit_mc(&empty[s], kBoth);
         }
         if (!ok) break;
-        umma_commit(&acc_full[acc]);     // the accumulator is complete
+        // the accumulator is complete (pair form: in both CTAs)
+        if constexpr (kPair) umma_commit_pair_mc(&acc_full[acc], kBoth);
+        else umma_commit(&acc_full[acc]);
       }
     }
     if (!ok) atomicExch(cta_err, 1);
@@ -244,7 +291,10 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&acc_empty[acc]);
+        if (lane == 0) {
+          if (kPair && rank != 0) mbar_arrive_cluster(cluster_addr(&acc_empty[acc], 0));
+          else mbar_arrive(&acc_empty[acc]);
+        }
       }
       if (ok && p.u_reduce && rows_exist) {
         // this run's share of the slot total
@@ -269,35 +319,48 @@ tc_grad_kernel(const __grid_constant__ CUtensorMap tmR, const __grid_constant__ 
     if (!ok) atomicExch(cta_err, 1);
   }
   __syncthreads();
-  cluster_sync_all();                    // no multicast or remote arrive is still aimed at this CTA
-  if (warp == 1) {
-    // every MMA of this CTA has completed before its accumulator was drained;
-    // after a failure, wait (bounded) for the last commits before releasing
-    if (*cta_err && lane == 0) {
-      int total = 0;
-      for (int i = 0; i < my_units; ++i) total += p.units[pair + i * npairs].w;
-      for (int a = 0; a < 2 && a < total; ++a) {
-        const int last = ((total - 1 - a) / 2) * 2 + a;
-        mbar_wait(&acc_full[a], (last / 2) & 1, p.status);
-      }
+  if (warp == 1 && lane == 0 && issuer && *cta_err) {
+    // every MMA has completed before its accumulator was drained; after a
+    // failure, wait (bounded) for the last commits before TMEM is released
+    int total = 0;
+    for (int i = 0; i < my_units; ++i) total += p.units[pair + i * npairs].w;
+    for (int a = 0; a < 2 && a < total; ++a) {
+      const int last = ((total - 1 - a) / 2) * 2 + a;
+      mbar_wait(&acc_full[a], (last / 2) & 1, p.status);
     }
-    __syncwarp();
+  }
+  __syncthreads();
+  cluster_sync_all();                    // no multicast, MMA or remote arrive is still aimed at this CTA
+  if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kGTmem) : "memory");
+    if constexpr (kPair)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kGTmem) : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kGTmem) : "memory");
   }
 }
 
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-static size_t grad_smem_bytes() { return 1024 + grad_smem().total; }
+template <bool kPair>
+static size_t grad_smem_bytes() { return 1024 + grad_smem<kPair>().total; }
 
-int tc_grad_max_pairs() {
-  static int mp = -1;
-  if (mp >= 0) return mp;
-  mp = 0;
-  const size_t smem = grad_smem_bytes();
-  if (cudaFuncSetAttribute(tc_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+// The pair form unless PGC_GRAD_PAIR_MMA=0 asks for the two-MMA form.
+static bool use_pair_mma() {
+  static int v = -1;
+  if (v < 0) {
+    const char* env = std::getenv("PGC_GRAD_PAIR_MMA");
+    v = (env && env[0] == '0') ? 0 : 1;
+  }
+  return v != 0;
+}
+
+template <bool kPair>
+static int max_pairs() {
+  const size_t smem = grad_smem_bytes<kPair>();
+  if (cudaFuncSetAttribute(tc_grad_kernel<kPair>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+      cudaSuccess)
     return 0;
   cudaLaunchConfig_t q = {};
   q.gridDim = dim3(2);
@@ -311,8 +374,13 @@ int tc_grad_max_pairs() {
   q.attrs = attr;
   q.numAttrs = 1;
   int nc = 0;
-  if (cudaOccupancyMaxActiveClusters(&nc, tc_grad_kernel, &q) != cudaSuccess) return 0;
-  mp = nc;
+  if (cudaOccupancyMaxActiveClusters(&nc, tc_grad_kernel<kPair>, &q) != cudaSuccess) return 0;
+  return nc;
+}
+
+int tc_grad_max_pairs() {
+  static int mp = -1;
+  if (mp < 0) mp = use_pair_mma() ? max_pairs<true>() : max_pairs<false>();
   return mp;
 }
 
@@ -320,8 +388,11 @@ cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, co
                            int npairs, cudaStream_t st) {
   if (p.nunits <= 0) return cudaSuccess;
   if (npairs < 1) return cudaErrorInvalidValue;
-  const size_t smem = grad_smem_bytes();
-  cudaError_t e = cudaFuncSetAttribute(tc_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const bool pair_mma = use_pair_mma();
+  const size_t smem = pair_mma ? grad_smem_bytes<true>() : grad_smem_bytes<false>();
+  cudaError_t e = pair_mma
+                      ? cudaFuncSetAttribute(tc_grad_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)
+                      : cudaFuncSetAttribute(tc_grad_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int pairs = npairs < p.nunits ? npairs : p.nunits;
   cudaLaunchConfig_t cfg = {};
@@ -343,7 +414,8 @@ cudaError_t launch_tc_grad(const void* tmR, const void* tmX, const void* tmU, co
   std::memcpy(&b, tmX, sizeof(CUtensorMap));
   std::memcpy(&u, tmU, sizeof(CUtensorMap));
   std::memcpy(&w, tmS, sizeof(CUtensorMap));
-  return cudaLaunchKernelEx(&cfg, tc_grad_kernel, a, b, u, w, p);
+  return pair_mma ? cudaLaunchKernelEx(&cfg, tc_grad_kernel<true>, a, b, u, w, p)
+                  : cudaLaunchKernelEx(&cfg, tc_grad_kernel<false>, a, b, u, w, p);
 }
 
 }  // namespace pgc
