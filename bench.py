@@ -121,7 +121,7 @@ def kernel_label(w: W.Workload, single: bool, dom: int) -> str:
     if tensor_core_path(w):
         nt = -(-w.K // 256)
         if dom == 2:
-            return "tc_grad_kernel, gradient R^T X (tcgen05, 2-CTA clusters, runs of partitions)"
+            return "tc_grad_kernel, gradient R^T X (tcgen05.mma.cta_group::2 over CTA pairs, runs of partitions)"
         if nt in (1, 2, 4, 8):
             return f"tc_logits_softmax_kernel, logits X W^T + softmax residual (tcgen05, {nt}-CTA clusters)"
         return "tc_gemm_kernel, logits X W^T (tcgen05, 2-CTA clusters)"
