@@ -540,7 +540,9 @@ def measure(w: W.Workload, K_steps: int, Wu: int, seed: int, mode: str, cpu_seco
     # workers' compute, the decode is the master's; seeded delays in units of
     # the compute time ------------------------------------------------------
     from paper_2607_20739_gb300 import wallclock as WC
-    decode_ms = min(group_ms[4], ms_per_step)
+    # (paths whose gradient kernel decodes in its own tail launch no decode
+    # kernel: their decode group holds only the events' own time)
+    decode_ms = min(group_ms[4], ms_per_step) if tim["launches"][4] > 0 else 0.0
     compute_ms = ms_per_step - decode_ms
     # one partition per worker: a GC run evaluates c partitions per worker
     compute_s = compute_ms * 1e-3 / (w.c if mode == "gc" else 1)
