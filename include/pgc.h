@@ -181,7 +181,11 @@ int pgc_load_partitions(pgc_ctx *ctx, const void *const *X, const void *const *y
  *   w_out          : [K*d] float32, receives beta^(t+1) (NULL: not returned).
  *   outputs_on_device : != 0: grad_out / w_out are device pointers and the
  *                    call returns without waiting for the GPU; 0: host
- *                    pointers, the call waits for the copies.
+ *                    pointers, the call waits until they hold the results
+ *                    (pinned host buffers mapped into the device's address
+ *                    space, 16-byte aligned, with d a multiple of the row
+ *                    padding, are written by the decode kernel itself;
+ *                    others are filled by copies after it).
  *   info           : may be NULL; receives t, o_t and the schedule indices.
  * Step 0 is the warm-up: every worker evaluates all c of its partitions at
  * beta^(0).  From step 1 on, worker W_i evaluates only the partition in its

@@ -435,6 +435,18 @@ void free_all(pgc_ctx* ctx) {
     if (p) cudaFree(p);
 }
 
+// Device address of a pinned host buffer mapped into the current device's
+// address space, or nullptr (pageable memory, or not addressable).
+void* mapped_host(const void* p) {
+  if (!p) return nullptr;
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();   // not a CUDA pointer: clear the error
+    return nullptr;
+  }
+  return at.type == cudaMemoryTypeHost ? at.devicePointer : nullptr;
+}
+
 int copy_out(pgc_ctx* ctx, float* dst, const float* src, int on_device) {
   // unpad [K][ld] -> [K][d]
   const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
@@ -844,11 +856,21 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
   dc.scheme = ctx->scheme; dc.n = n; dc.s = ctx->s; dc.c = c; dc.slot = ph.slot; dc.owners = ctx->owners;
   dc.mask = bits; dc.P = ctx->P; dc.store = ctx->store; dc.U = ctx->U; dc.w = ctx->w; dc.wb = ctx->wb;
   dc.gout = ctx->gout; dc.lr = ctx->lr; dc.coeff_out = ctx->coeff; dc.status = ctx->status;
-  // device outputs with the unpadded layout (ld == d) and 16-byte alignment are
-  // written by the decode itself, so no copy sits between consecutive steps
-  const bool direct = outputs_on_device && ctx->ld == ctx->d &&
-                      (reinterpret_cast<uintptr_t>(grad_out) % 16 == 0) && (reinterpret_cast<uintptr_t>(w_out) % 16 == 0);
-  if (direct) { dc.g_user = grad_out; dc.w_user = w_out; }
+  // outputs with the unpadded layout (ld == d) and 16-byte alignment that the
+  // GPU can address are written by the decode itself: device outputs (so no
+  // copy sits between consecutive steps), and pinned host outputs mapped into
+  // the device's address space (so no device-to-host copies follow the decode)
+  float* g_dev = grad_out;
+  float* w_dev = w_out;
+  bool direct = ctx->ld == ctx->d && (reinterpret_cast<uintptr_t>(grad_out) % 16 == 0) &&
+                (reinterpret_cast<uintptr_t>(w_out) % 16 == 0);
+  if (direct && !outputs_on_device) {
+    g_dev = static_cast<float*>(mapped_host(grad_out));
+    w_dev = static_cast<float*>(mapped_host(w_out));
+    direct = (!grad_out || g_dev) && (!w_out || w_dev) && (reinterpret_cast<uintptr_t>(g_dev) % 16 == 0) &&
+             (reinterpret_cast<uintptr_t>(w_dev) % 16 == 0);
+  }
+  if (direct) { dc.g_user = g_dev; dc.w_user = w_dev; }
   bool need_commit = true, need_decode = true;
   if (ctx->loss != PGC_SOFTMAX) {
     // K1 with its fused tail: commit (and, for small P, decode) in the same launch
