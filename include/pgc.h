@@ -183,8 +183,8 @@ int pgc_load_partitions(pgc_ctx *ctx, const void *const *X, const void *const *y
  *                    call returns without waiting for the GPU; 0: host
  *                    pointers, the call waits until they hold the results
  *                    (pinned host buffers mapped into the device's address
- *                    space, 16-byte aligned, with d a multiple of the row
- *                    padding, are written by the decode kernel itself;
+ *                    space and 16-byte aligned are written by the decode
+ *                    kernel itself when the parameter rows need no padding;
  *                    others are filled by copies after it).
  *   info           : may be NULL; receives t, o_t and the schedule indices.
  * Step 0 is the warm-up: every worker evaluates all c of its partitions at
