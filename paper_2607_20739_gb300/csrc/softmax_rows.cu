@@ -27,11 +27,12 @@
 //      operand of the gradient MMA) and release the slot, so a slot is held
 //      only for its load, the logits and the copy, not for the exchange of
 //      step 2; kNA copies (and R blocks) rotate;
-//   4. one thread issues tcgen05.mma (M = 128 features, N = 16 classes, K =
-//      the 16 rows; A = the tile's copy in tensor memory, B = R_hi, then
-//      again with B = R_lo) into a TMEM
-//      accumulator of the CTA's half of G^T that spans the pair's run of tiles
-//      in a partition; its commit frees the copy and the R block.
+//   4. two threads, each for half of the 128-feature slices, issue
+//      tcgen05.mma (M = 128 features, N = 16 classes, K = the 16 rows; A =
+//      the tile's copy in tensor memory, B = R_hi, then again with B = R_lo)
+//      into a TMEM accumulator of the CTA's half of G^T that spans the pair's
+//      run of tiles in a partition; their two commits free the copy and the
+//      R block.
 // No data leaves the pair before the end of a run; then the eight warps write
 // the run's G^T halves into one partial (one item per pair and partition).
 // With the fused tail the same grid then commits and decodes: after a grid
@@ -58,7 +59,8 @@ constexpr int kPairCtas = 2;             // CTAs per cluster: feature halves
 constexpr int kFw = 8;                   // forward warps (warps 2..9)
 constexpr int kRWarp = 2 + kFw;          // the residual warps (even and odd tiles)
 constexpr int kNRes = 2;
-constexpr int kRThreads = 64 + 32 * kFw + 32 * kNRes;
+constexpr int kMWarp2 = kRWarp + kNRes;  // the second MMA-issuing warp (warp 1 is the first)
+constexpr int kRThreads = 64 + 32 * kFw + 32 * kNRes + 32;
 // 16-feature steps per forward warp at the largest ld
 constexpr int kMaxKs = (int)(kRowsMaxLd / kPairCtas / (16 * kFw));
 constexpr uint32_t kZp = kRR * 16 * 4;   // a 16 x 16 fp32 block of partial logits
@@ -270,7 +272,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     for (int b = 0; b < kNA; ++b) {
       mbar_init(&rready[b], 1);
       mbar_init(&a_full[b], kFw);
-      mbar_init(&a_empty[b], 1);
+      mbar_init(&a_empty[b], 2);         // the commits of both MMA issuers
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&zready[b], kFw);
@@ -278,7 +280,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       mbar_init(&zpeer_full[b], 1);
       mbar_init(&zpeer_empty[b], 1);
     }
-    mbar_init(acc_full, 1);
+    mbar_init(acc_full, 2);
     mbar_init(acc_empty, kFw);
     fence_mbar_init();
   }
@@ -319,9 +321,14 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       const int last = ((issued - 1 - s) / S) * S + s;
       mbar_wait(&full[s], (last / S) & 1, a.status);
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if ((warp == 1 || warp == kMWarp2) && lane == 0) {
     // ---- backward MMAs: G^T[f][k] += sum_r X[r][f] R[r][k] ------------------
+    // Two issuing threads, each with half of the 128-feature slices (they
+    // write different accumulator columns): a single thread issues these
+    // small MMAs more slowly than the tiles arrive.  Each commits its own
+    // MMAs; the barriers they free count both.
     constexpr uint32_t id_bwd = idesc_bf16_f32(128, 16, false, false);
+    const int mt0 = warp == 1 ? 0 : (nmt + 1) / 2, mt1 = warp == 1 ? (nmt + 1) / 2 : nmt;
     bool ok = true;
     int run = 0;
     for (int i = 0; i < n && ok; ++i) {
@@ -338,14 +345,14 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       const uint64_t dbl = sdesc(smem_u32(rblk + (kNA + ab) * kRb), 256, 128, 0);
       // slice mt: its 128 features x 16 rows are columns kAccCols + ab kAStride + 8 mt ..
       const uint32_t ta = tmem + kAccCols + (uint32_t)ab * kAStride;
-      // all slices with R_hi, then all with R_lo: consecutive MMAs write
-      // different accumulators
-      for (int mt = 0; mt < nmt; ++mt) {
+      // all of this issuer's slices with R_hi, then with R_lo: consecutive
+      // MMAs write different accumulators
+      for (int mt = mt0; mt < mt1; ++mt) {
         const uint32_t d = tmem + (uint32_t)(mt * 16), am = ta + (uint32_t)(mt * 8);
         if (first) umma_ta_fresh(d, am, db, id_bwd);
         else umma_ta_acc(d, am, db, id_bwd);
       }
-      for (int mt = 0; mt < nmt; ++mt) umma_ta_acc(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), dbl, id_bwd);
+      for (int mt = mt0; mt < mt1; ++mt) umma_ta_acc(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), dbl, id_bwd);
       umma_commit(&a_empty[ab]);
       if (last) {
         umma_commit(acc_full);
@@ -353,7 +360,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       }
     }
     if (!ok) atomicExch(cta_err, 1);
-  } else if (warp >= kRWarp) {
+  } else if (warp >= kRWarp && warp < kRWarp + kNRes) {
     // ---- residual: the pair's logits, R = softmax(Z) - onehot(y) ------------
     // Two warps, for the even and the odd tiles (every buffer and barrier of
     // the exchange is per tile parity), so one tile's exchange with the other
@@ -444,7 +451,7 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       if (lane == 0) mbar_arrive(&rready[i % kNA]);
     }
     if (!ok) atomicExch(cta_err, 1);
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp < kRWarp) {
     // ---- forward (8 warps), run drain (all 8) ---------------------------------
     const int fw = warp - 2;
     const int nks = (int)(ldh / (16 * kFw));    // 16-feature steps of this warp
