@@ -17,11 +17,13 @@
 //      16 x 16 block to the other CTA with st.async into distributed shared
 //      memory, add the two blocks in rank order (so both CTAs form the same
 //      R) and form R = softmax(Z) - onehot(y) (zero past K and past the
-//      partition's rows) as two bf16 blocks, R_hi = bf16(R) and R_lo =
-//      bf16(R - R_hi), in the no-swizzle K-major operand layout (R alone in
-//      bf16 is not enough: when the rows' softmax values are alike, their
-//      rounding errors are alike too and add up coherently over the rows of
-//      the contraction with non-negative features);
+//      partition's rows) in bf16, in the no-swizzle K-major operand layout.
+//      The rounding uses error feedback: each entry's rounding error is
+//      added to the same entry (row position, class) of the warp's next tile
+//      of the run before that one is rounded, so over a run the errors
+//      telescope instead of adding up.  Rounded independently, entries of
+//      rows with alike softmax values round alike, and with non-negative
+//      features those errors add up coherently over the rows of R^T X;
 //   3. the same eight warps copy the half tile, transposed, into tensor memory
 //      (one lane per feature, two rows per 32-bit column: the K-major A
 //      operand of the gradient MMA) and release the slot, so a slot is held
@@ -29,10 +31,9 @@
 //      step 2; kNA copies (and R blocks) rotate;
 //   4. two threads, each for half of the 128-feature slices, issue
 //      tcgen05.mma (M = 128 features, N = 16 classes, K = the 16 rows; A =
-//      the tile's copy in tensor memory, B = R_hi, then again with B = R_lo)
-//      into a TMEM accumulator of the CTA's half of G^T that spans the pair's
-//      run of tiles in a partition; their two commits free the copy and the
-//      R block.
+//      the tile's copy in tensor memory, B = the R block) into a TMEM
+//      accumulator of the CTA's half of G^T that spans the pair's run of
+//      tiles in a partition; their two commits free the copy and the R block.
 // No data leaves the pair before the end of a run; then the eight warps write
 // the run's G^T halves into one partial (one item per pair and partition).
 // With the fused tail the same grid then commits and decodes: after a grid
@@ -64,8 +65,9 @@ constexpr int kRThreads = 64 + 32 * kFw + 32 * kNRes + 32;
 // 16-feature steps per forward warp at the largest ld
 constexpr int kMaxKs = (int)(kRowsMaxLd / kPairCtas / (16 * kFw));
 constexpr uint32_t kZp = kRR * 16 * 4;   // a 16 x 16 fp32 block of partial logits
-constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16); R_lo blocks follow the kNA R_hi
+constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16)
 constexpr int kNA = 3;                   // tiles whose gradient MMA may be pending (TMEM copies, R blocks)
+constexpr int kTailMaxC = 4;             // slots per store on the fused tail's short route
 constexpr int kTmemCols = 512;           // G^T half, then the kNA copies of a tile
 constexpr uint32_t kAccCols = 192;       // G^T half: ld / 256 slices of 16 columns at the largest ld
 constexpr uint32_t kAStride = 96;        // a copy: ld / 256 slices of 8 columns (16 rows of bf16)
@@ -210,8 +212,7 @@ __device__ bool grid_barrier(int* ctr, int* status, int* flag) {
 
 // Shared memory of a CTA: slots of its half tile, two sets (tile parity) of
 // the forward warps' partial logits (the fused tail's decode plan reuses
-// them), two blocks for the other CTA's partial, kNA R_hi then kNA R_lo
-// blocks, barriers.
+// them), two blocks for the other CTA's partial, kNA R blocks, barriers.
 struct RowsSmem {
   uint32_t slot_bytes, zpart, zpeer, rblk, bars, total;
 };
@@ -222,7 +223,7 @@ __host__ __device__ static RowsSmem rows_smem(int64_t ld, int nslots) {
   s.zpart = (uint32_t)nslots * s.slot_bytes;
   s.zpeer = s.zpart + 2 * kFw * kZp;
   s.rblk = s.zpeer + 2 * kZp;
-  s.bars = s.rblk + 2u * (uint32_t)kNA * kRb;
+  s.bars = s.rblk + (uint32_t)kNA * kRb;
   s.total = s.bars + kRowsBars * 8 + 16;
   return s;
 }
@@ -342,17 +343,13 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
       if (first && run > 0 && !mbar_wait(acc_empty, (run - 1) & 1, a.status)) { ok = false; break; }
       tc_fence_after();
       const uint64_t db = sdesc(smem_u32(rblk + ab * kRb), 256, 128, 0);
-      const uint64_t dbl = sdesc(smem_u32(rblk + (kNA + ab) * kRb), 256, 128, 0);
       // slice mt: its 128 features x 16 rows are columns kAccCols + ab kAStride + 8 mt ..
       const uint32_t ta = tmem + kAccCols + (uint32_t)ab * kAStride;
-      // all of this issuer's slices with R_hi, then with R_lo: consecutive
-      // MMAs write different accumulators
       for (int mt = mt0; mt < mt1; ++mt) {
         const uint32_t d = tmem + (uint32_t)(mt * 16), am = ta + (uint32_t)(mt * 8);
         if (first) umma_ta_fresh(d, am, db, id_bwd);
         else umma_ta_acc(d, am, db, id_bwd);
       }
-      for (int mt = mt0; mt < mt1; ++mt) umma_ta_acc(tmem + (uint32_t)(mt * 16), ta + (uint32_t)(mt * 8), dbl, id_bwd);
       umma_commit(&a_empty[ab]);
       if (last) {
         umma_commit(acc_full);
@@ -366,14 +363,22 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     // the exchange is per tile parity), so one tile's exchange with the other
     // CTA overlaps the next tile's.  lane: row lane / 2, classes 8 (lane & 1)
     // .. + 7.  The R block i % kNA is written once tile i - kNA's MMAs have
-    // read it (a_empty).
+    // read it (a_empty).  ef: the rounding errors of this lane's entries in
+    // the warp's previous tile of the same run (error feedback).
     const int r = lane >> 1, kh = (lane & 1) * 8;
     const uint32_t peer = (uint32_t)(rank ^ 1);
     bool ok = true;
+    float ef[8];
+    int ef_item = -1;
     for (int i = warp - kRWarp; i < n && ok; i += kNRes) {
       const int b = i & 1;
       const int4 tl = a.tiles[t0 + i];
       const bool valid = r < tl.y;
+      if (tl.z != ef_item) {                             // a new run: nothing carried in
+        ef_item = tl.z;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) ef[c] = 0.f;
+      }
       const int lab = valid ? a.y[tl.x + r] : -1;        // fetched before the waits
       if (!__all_sync(0xffffffffu, mbar_wait(&zready[b], (i >> 1) & 1, a.status))) { ok = false; break; }
       float z[8];
@@ -436,15 +441,16 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
         break;
       }
       uint8_t* blk = rblk + (i % kNA) * kRb;
-      uint8_t* blk_lo = rblk + (kNA + i % kNA) * kRb;
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         const int k = kh + c;
-        const float v = valid && k < a.K ? e[c] * inv - (k == lab ? 1.f : 0.f) : 0.f;
-        const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-        const uint32_t off = r_offset(k, k_of_row(r));
-        *reinterpret_cast<__nv_bfloat16*>(blk + off) = hi;
-        *reinterpret_cast<__nv_bfloat16*>(blk_lo + off) = __float2bfloat16_rn(v - __bfloat162float(hi));
+        __nv_bfloat16 q = __float2bfloat16_rn(0.f);
+        if (valid && k < a.K) {
+          const float v = e[c] * inv - (k == lab ? 1.f : 0.f) + ef[c];
+          q = __float2bfloat16_rn(v);
+          ef[c] = v - __bfloat162float(q);
+        }
+        *reinterpret_cast<__nv_bfloat16*>(blk + r_offset(k, k_of_row(r))) = q;
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -611,9 +617,28 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
     // decodes that slice: a column's decode reads only that column of the
     // stores and slot totals, all written by this CTA, so a CTA barrier
     // stands in for a second grid barrier.
+    //
+    // Steady steps (one store per evaluated partition, every store's slot o_t
+    // refreshed) take a shorter route: the slot totals this step leaves as
+    // they are, and beta, are loaded before the grid barrier, and the
+    // committed gradients reach the decode through shared memory (the slots'
+    // area, idle after the tiles), so U[o_t] = sum_e g_e needs no second
+    // round trip through L2.
     if (warp == 0) derive_plan_warp(a.dec, plan, lane);   // needs only the mask
     const int64_t P4 = a.P / 4;
     const int64_t q0 = P4 * blockIdx.x / gridDim.x, q1 = P4 * (blockIdx.x + 1) / gridDim.x, nq = q1 - q0;
+    const DecodeArgs& dc = a.dec;
+    const bool fast = dc.slot >= 0 && !dc.u_ready && a.ndest == 1 && a.nE == dc.owners && dc.c <= kTailMaxC &&
+                      nq <= (int64_t)blockDim.x && (int64_t)a.nE * nq * 16 <= (int64_t)S * L.slot_bytes;
+    float4* gs = reinterpret_cast<float4*>(sm);           // [nE][nq] committed gradients (fast route)
+    float4 up[kTailMaxC], wv = f4zero();
+    const int64_t pq = q0 + threadIdx.x;
+    if (fast && (int64_t)threadIdx.x < nq) {
+      const float4* U4 = reinterpret_cast<const float4*>(dc.U);
+#pragma unroll
+      for (int o = 0; o < kTailMaxC; ++o) up[o] = (o < dc.c && o != dc.slot) ? __ldcg(U4 + (int64_t)o * P4 + pq) : f4zero();
+      wv = __ldcg(reinterpret_cast<const float4*>(dc.w) + pq);
+    }
     bool ok = grid_barrier(a.counters, a.status, &bar_flag);   // every partial is written
     if (ok) {
       const float4* src = reinterpret_cast<const float4*>(a.partials);
@@ -637,10 +662,30 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
           const int dst = a.e_dest[(int64_t)e * a.ndest + k];
           if (dst >= 0) reinterpret_cast<float4*>(a.store)[(int64_t)dst * P4 + p] = acc;
         }
+        if (fast) gs[x] = acc;
       }
-      __syncthreads();                   // this CTA's stores are visible to all its threads
+      __syncthreads();                   // this CTA's stores (and gs) are visible to all its threads
       if (blockIdx.x == 0 && warp == 0) write_coeffs_warp(a.dec, lane);
-      decode_columns(a.dec, plan, q0, q1, (int)threadIdx.x, (int)blockDim.x);
+      if (!fast) {
+        decode_columns(a.dec, plan, q0, q1, (int)threadIdx.x, (int)blockDim.x);
+      } else if ((int64_t)threadIdx.x < nq) {
+        // U[o_t] = sum over the evaluated partitions of their new gradients
+        float4 un = f4zero();
+        for (int e = 0; e < a.nE; ++e) un = f4add(un, gs[(int64_t)e * nq + threadIdx.x]);
+        reinterpret_cast<float4*>(dc.U)[(int64_t)dc.slot * P4 + pq] = un;
+        float4 V = f4zero(), D = f4zero();
+#pragma unroll
+        for (int o = 0; o < kTailMaxC; ++o)
+          if (o < dc.c) V = f4add(V, o == dc.slot ? un : up[o]);
+        const float4* st4 = reinterpret_cast<const float4*>(dc.store);
+        for (int q = 0; q < plan.ndev; ++q) {
+          float4 Cr = f4zero();
+          for (int o = 0; o < dc.c; ++o) Cr = f4add(Cr, __ldcg(st4 + ((int64_t)plan.dev[q] * dc.c + o) * P4 + pq));
+          D = f4fma(plan.devc[q], Cr, D);
+        }
+        const float4 g = f4fma(plan.B, V, D);
+        store_outputs(dc, pq, g, f4fma(-dc.lr, g, wv));
+      }
       __syncthreads();
       // the last CTA out resets the counters for the next step
       if (threadIdx.x == 0 && atomic_add_acq_rel(a.counters + 2, 1) == (int)gridDim.x - 1) {
