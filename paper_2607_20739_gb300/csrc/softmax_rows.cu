@@ -47,6 +47,7 @@
 
 #include <cstring>
 
+#include "rows_tail.cuh"
 #include "tc_common.cuh"
 
 namespace pgc {
@@ -67,7 +68,6 @@ constexpr int kMaxKs = (int)(kRowsMaxLd / kPairCtas / (16 * kFw));
 constexpr uint32_t kZp = kRR * 16 * 4;   // a 16 x 16 fp32 block of partial logits
 constexpr uint32_t kRb = 16 * 16 * 2;    // R block (16 rows x 16 classes bf16)
 constexpr int kNA = 3;                   // tiles whose gradient MMA may be pending (TMEM copies, R blocks)
-constexpr int kTailMaxC = 4;             // slots per store on the fused tail's short route
 constexpr int kTmemCols = 512;           // G^T half, then the kNA copies of a tile
 constexpr uint32_t kAccCols = 192;       // G^T half: ld / 256 slices of 16 columns at the largest ld
 constexpr uint32_t kAStride = 96;        // a copy: ld / 256 slices of 8 columns (16 rows of bf16)
@@ -177,37 +177,6 @@ __device__ __forceinline__ bool wait_cluster(uint64_t* bar, uint32_t parity, int
 __device__ __forceinline__ uint32_t r_offset(int k, int r) {
   return (uint32_t)((r >> 3) * 256 + (k >> 3) * 128 + (k & 7) * 16 + (r & 7) * 2);
 }
-__device__ __forceinline__ int ld_acquire(const int* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-// Every CTA of the (co-resident) grid arrives on *ctr and waits until all
-// have; bounded.  Called by all threads of the CTA.
-__device__ bool grid_barrier(int* ctr, int* status, int* flag) {
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int ok = 1;
-    atomic_add_acq_rel(ctr, 1);
-    const int target = (int)gridDim.x;
-    if (ld_acquire(ctr) < target) {
-      const uint64_t t0 = globaltimer_ns();
-      for (uint32_t it = 0;; ++it) {
-        if (ld_acquire(ctr) >= target) break;
-        if (it > kWaitMaxIters || ((it & 63u) == 63u && globaltimer_ns() - t0 > kWaitMaxNs)) {
-          atomicOr(status, kErrWaitTimeout);
-          ok = 0;
-          break;
-        }
-      }
-    }
-    *flag = ok;
-  }
-  __syncthreads();
-  return *flag != 0;
-}
-
 }  // namespace
 
 // Shared memory of a CTA: slots of its half tile, two sets (tile parity) of
@@ -611,89 +580,10 @@ softmax_rows_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_consta
   cluster_sync_all();                    // no st.async or remote arrive is still aimed at this CTA
   tc_fence_after();
   if (a.tail && !*cta_err) {
-    // ---- fused tail: commit, then decode + SGD --------------------------------
-    // After one grid barrier (every partial written) each CTA commits every
-    // evaluated partition for its own slice of the float4 columns and then
-    // decodes that slice: a column's decode reads only that column of the
-    // stores and slot totals, all written by this CTA, so a CTA barrier
-    // stands in for a second grid barrier.
-    //
-    // Steady steps (one store per evaluated partition, every store's slot o_t
-    // refreshed) take a shorter route: the slot totals this step leaves as
-    // they are, and beta, are loaded before the grid barrier, and the
-    // committed gradients reach the decode through shared memory (the slots'
-    // area, idle after the tiles), so U[o_t] = sum_e g_e needs no second
-    // round trip through L2.
-    if (warp == 0) derive_plan_warp(a.dec, plan, lane);   // needs only the mask
-    const int64_t P4 = a.P / 4;
-    const int64_t q0 = P4 * blockIdx.x / gridDim.x, q1 = P4 * (blockIdx.x + 1) / gridDim.x, nq = q1 - q0;
-    const DecodeArgs& dc = a.dec;
-    const bool fast = dc.slot >= 0 && !dc.u_ready && a.ndest == 1 && a.nE == dc.owners && dc.c <= kTailMaxC &&
-                      nq <= (int64_t)blockDim.x && (int64_t)a.nE * nq * 16 <= (int64_t)S * L.slot_bytes;
-    float4* gs = reinterpret_cast<float4*>(sm);           // [nE][nq] committed gradients (fast route)
-    float4 up[kTailMaxC], wv = f4zero();
-    const int64_t pq = q0 + threadIdx.x;
-    if (fast && (int64_t)threadIdx.x < nq) {
-      const float4* U4 = reinterpret_cast<const float4*>(dc.U);
-#pragma unroll
-      for (int o = 0; o < kTailMaxC; ++o) up[o] = (o < dc.c && o != dc.slot) ? __ldcg(U4 + (int64_t)o * P4 + pq) : f4zero();
-      wv = __ldcg(reinterpret_cast<const float4*>(dc.w) + pq);
-    }
-    bool ok = grid_barrier(a.counters, a.status, &bar_flag);   // every partial is written
-    if (ok) {
-      const float4* src = reinterpret_cast<const float4*>(a.partials);
-      for (int64_t x = threadIdx.x; x < (int64_t)a.nE * nq; x += blockDim.x) {
-        const int e = (int)(x / nq);
-        const int64_t p = q0 + (x - (int64_t)e * nq);
-        const int i0 = a.e_item0[e], i1 = a.e_item0[e + 1];
-        float4 acc = f4zero();
-        // a partition has about (pairs / partitions) + 1 items: one batch of
-        // loads in flight covers it
-        for (int it = i0; it < i1; it += 16) {
-          float4 v[16];
-#pragma unroll
-          for (int u = 0; u < 16; ++u) v[u] = it + u < i1 ? __ldcg(src + (int64_t)(it + u) * P4 + p) : f4zero();
-#pragma unroll
-          for (int u = 0; u < 16; ++u) acc = f4add(acc, v[u]);
-        }
-        const float sc = a.e_scale[e];
-        acc = make_float4(acc.x * sc, acc.y * sc, acc.z * sc, acc.w * sc);
-        for (int k = 0; k < a.ndest; ++k) {
-          const int dst = a.e_dest[(int64_t)e * a.ndest + k];
-          if (dst >= 0) reinterpret_cast<float4*>(a.store)[(int64_t)dst * P4 + p] = acc;
-        }
-        if (fast) gs[x] = acc;
-      }
-      __syncthreads();                   // this CTA's stores (and gs) are visible to all its threads
-      if (blockIdx.x == 0 && warp == 0) write_coeffs_warp(a.dec, lane);
-      if (!fast) {
-        decode_columns(a.dec, plan, q0, q1, (int)threadIdx.x, (int)blockDim.x);
-      } else if ((int64_t)threadIdx.x < nq) {
-        // U[o_t] = sum over the evaluated partitions of their new gradients
-        float4 un = f4zero();
-        for (int e = 0; e < a.nE; ++e) un = f4add(un, gs[(int64_t)e * nq + threadIdx.x]);
-        reinterpret_cast<float4*>(dc.U)[(int64_t)dc.slot * P4 + pq] = un;
-        float4 V = f4zero(), D = f4zero();
-#pragma unroll
-        for (int o = 0; o < kTailMaxC; ++o)
-          if (o < dc.c) V = f4add(V, o == dc.slot ? un : up[o]);
-        const float4* st4 = reinterpret_cast<const float4*>(dc.store);
-        for (int q = 0; q < plan.ndev; ++q) {
-          float4 Cr = f4zero();
-          for (int o = 0; o < dc.c; ++o) Cr = f4add(Cr, __ldcg(st4 + ((int64_t)plan.dev[q] * dc.c + o) * P4 + pq));
-          D = f4fma(plan.devc[q], Cr, D);
-        }
-        const float4 g = f4fma(plan.B, V, D);
-        store_outputs(dc, pq, g, f4fma(-dc.lr, g, wv));
-      }
-      __syncthreads();
-      // the last CTA out resets the counters for the next step
-      if (threadIdx.x == 0 && atomic_add_acq_rel(a.counters + 2, 1) == (int)gridDim.x - 1) {
-        a.counters[0] = 0;
-        a.counters[2] = 0;
-        __threadfence();
-      }
-    }
+    // ---- fused tail: commit, then decode + SGD (rows_tail.cuh); the decode
+    // plan goes where the partial logits were, the committed gradients of
+    // the short route where the slots were
+    rows_fused_tail(a, *reinterpret_cast<DecodePlan*>(zpart), sm, (int64_t)S * L.slot_bytes, &bar_flag);
   }
   if (warp == 1) {
     // after a failure, wait (bounded) for the last commit before releasing TMEM
