@@ -225,7 +225,7 @@ const char *pgc_strerror(int32_t code);
  * per-partition gradients with (fixed at pgc_create): "grad_rows" (logistic,
  * least squares), "tc_fused" (softmax on the tensor cores, residual in the
  * logits GEMM), "tc" (tensor cores, separate residual kernel),
- * "softmax_rows" (few classes, whole rows per CTA), "softmax_cluster" (few
+ * "softmax_rows" (few classes, whole rows per CTA pair), "softmax_cluster" (few
  * classes, 8-CTA clusters), "softmax_cc" (CUDA cores); "" for NULL. */
 const char *pgc_gradient_path(const pgc_ctx *ctx);
 
