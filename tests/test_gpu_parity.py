@@ -44,11 +44,15 @@ CASES = {
     # (six 256-class tiles: the three-kernel path)
     "cr_tc_k2000_nt8": (WL["cr_n128_softmax_k1000"].replace(n=3, s=1, K=2000, d=300, m=150), 4),
     "fr_tc_k1500_unfused": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=1500, d=256, m=(90, 200, 3, 128)), 4),
-    # few-class softmax (one-pass cluster kernel): ragged tiles, partition
+    # few-class softmax (whole-row kernel on CTA pairs): ragged tiles, partition
     # boundaries inside a cluster's run, empty feature slices, K = 16
     "fr_smallk_k10_unequal_rows": (WL["fr_n32_softmax_k10"].replace(n=4, s=1, d=3072, m=(300, 1, 129, 700)), 5),
     "cr_smallk_k16_d1000": (WL["fr_n32_softmax_k10"].replace(scheme="CR", n=6, s=2, K=16, d=1000, m=257), 5),
     "cr_smallk_k5_d64": (WL["fr_n32_softmax_k10"].replace(scheme="CR", n=5, s=1, K=5, d=64, m=(1, 2, 128, 129, 40)), 5),
+    # more slots per store (c = 6) than the fused tail's short route takes:
+    # its decode reads the stores and slot totals back from L2; ten steps
+    # cover every slot after the warm-up
+    "cr_smallk_c6_k10_d256": (WL["fr_n32_softmax_k10"].replace(scheme="CR", n=8, s=5, K=10, d=256, m=(40, 97, 1, 64, 33, 120, 8, 71)), 10),
     # P = K d >= 2^20: the one-thread-per-column decode
     "cr_tc_wide_decode": (WL["cr_n128_softmax_k1000"].replace(n=5, s=2, K=256, d=4096, m=64), 5),
     "fr_tc_wide_decode": (WL["cr_n128_softmax_k1000"].replace(scheme="FR", n=4, s=1, K=300, d=4000, m=(70, 129, 1, 64)), 5),
@@ -238,6 +242,7 @@ EXPECTED_PATHS = {
     "fr_bf16_softmax_k2": "softmax_rows",
     "fr_smallk_k10_unequal_rows": "softmax_rows",
     "cr_smallk_k16_d1000": "softmax_rows",
+    "cr_smallk_c6_k10_d256": "softmax_rows",
     "cr_tc_k300_d320_m200": "tc_fused",
     "cr_tc_k2000_nt8": "tc_fused",
     "fr_tc_k1500_unfused": "tc",
