@@ -111,6 +111,27 @@ __global__ void __launch_bounds__(256) decode_wide_kernel(DecodeArgs a) {
   const float4* store = reinterpret_cast<const float4*>(a.store);
   float4* U = reinterpret_cast<float4*>(a.U);
   const int64_t slotP = (int64_t)c * P4;           // float4s per store
+  if (a.pre && a.u_ready && a.slot >= 0) {
+    // the slots other than o_t were summed early: add U[o_t] and the
+    // deviating stores' slot o_t
+    const float4* pre = reinterpret_cast<const float4*>(a.pre);
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P4; p += (int64_t)gridDim.x * blockDim.x) {
+      float4 g = f4fma(pl.B, __ldcg(U + (int64_t)a.slot * P4 + p), __ldcg(pre + p));
+      const float4* cur = store + (int64_t)a.slot * P4 + p;
+      for (int q0 = 0; q0 < pl.ndev; q0 += 8) {
+        float4 v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = q0 + j < pl.ndev ? __ldcg(cur + (int64_t)pl.dev[q0 + j] * slotP) : f4zero();
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          if (q0 + j < pl.ndev) g = f4fma(pl.devc[q0 + j], v[j], g);
+      }
+      float4 w = __ldcg(reinterpret_cast<const float4*>(a.w) + p);
+      w = f4fma(-a.lr, g, w);
+      store_outputs(a, p, g, w);
+    }
+    return;
+  }
   for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < P4; p += (int64_t)gridDim.x * blockDim.x) {
     float4 V = f4zero();
     if (a.slot < 0) {

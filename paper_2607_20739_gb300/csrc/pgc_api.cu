@@ -139,6 +139,7 @@ struct pgc_ctx {
   alignas(64) unsigned char tmW16[128];  // Wb [16][ld] for the few-class kernel (box 64 x 16)
   int64_t Ktc = 0;           // classes padded to the forward N tile (256)
   uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]
+  float* pre = nullptr;      // fused tensor-core path: the decode's early terms [P]
   alignas(64) unsigned char tmXk[128];   // X as K-major A   (box 64 x 128)
   alignas(64) unsigned char tmW[128];    // Wb as K-major B  (box 64 x 128: one CTA's half of a 256 tile)
   alignas(64) unsigned char tmR[128];    // R as MN-major A  (box 64 x 64)
@@ -430,7 +431,7 @@ void free_all(pgc_ctx* ctx) {
   ctx->ev_pool.clear();
   void* ptrs[] = {ctx->X, ctx->y, ctx->w, ctx->wb, ctx->store, ctx->U, ctx->gout, ctx->partials, ctx->Z,
                   ctx->coeff, ctx->status, ctx->loss_blocks, ctx->loss_out, ctx->tables, ctx->counters, ctx->Rb,
-                  ctx->gc_coeff, ctx->gc_d, ctx->gc_draws, ctx->gc_wts};
+                  ctx->gc_coeff, ctx->gc_d, ctx->gc_draws, ctx->gc_wts, ctx->pre};
   for (void* p : ptrs)
     if (p) cudaFree(p);
 }
@@ -704,6 +705,12 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     PGC_ALLOC(ctx->Z, std::max(zcc, ztc) * sizeof(float));
   }
   if (ctx->tc) PGC_ALLOC(ctx->Rb, (size_t)max_zpad * ctx->Ktc * sizeof(uint16_t));
+  // the early decode terms run in the fused logits kernel when the decode
+  // reads enough to pay for it (the one-thread-per-column decode sizes);
+  // PGC_NO_PRE_DECODE=1 leaves the whole decode after the contraction
+  if (ctx->tc && ctx->tcf && !gc_weighted && ctx->P / 4 >= kPreDecodeMinP4 && s <= kPreMaxDev &&
+      !(std::getenv("PGC_NO_PRE_DECODE") && std::getenv("PGC_NO_PRE_DECODE")[0] == '1'))
+    PGC_ALLOC(ctx->pre, Pb);
   PGC_ALLOC(ctx->coeff, (size_t)n * sizeof(float));
   PGC_ALLOC(ctx->status, sizeof(int));
   PGC_ALLOC(ctx->loss_blocks, (size_t)ctx->loss_nblocks * sizeof(double));
@@ -909,6 +916,12 @@ int pgc_step(pgc_ctx* ctx, const uint8_t* mask, float* grad_out, float* w_out, i
       q.y = static_cast<const int32_t*>(ctx->y);
       q.zero_buf = u_red ? ctx->U + (size_t)ph.slot * ctx->P : nullptr; q.zero_n4 = ctx->P / 4;
       q.status = ctx->status; q.pdl = ctx->pdl ? 1 : 0;
+      if (u_red && ctx->pre) {
+        // the decode's terms of the slots other than o_t, summed beside the GEMM
+        q.pre = dc;
+        q.pre_out = ctx->pre;
+        dc.pre = ctx->pre;
+      }
       PGC_CK(ctx, launch_tc_softmax(ctx->tmXq, ctx->tmW, ctx->tmRst, q, ctx->tcf_nc, st));
       PGC_CK(ctx, record_event(ctx));
       PGC_CK(ctx, record_event(ctx));   // empty residual group

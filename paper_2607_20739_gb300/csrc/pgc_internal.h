@@ -51,6 +51,8 @@ struct DecodeArgs {
   float* g_user = nullptr;  // optional extra destinations of ghat and beta, same
   float* w_user = nullptr;  // unpadded layout (used when ld == d)
   int u_ready = 0;          // U[slot] already holds this step's slot total
+  const float* pre = nullptr;  // with u_ready: the terms of the slots other than o_t, summed
+                               // early (TcSoftmaxParams::pre_out)
 };
 // ---- K1: streaming gradient of logistic / least-squares partitions -------
 // For every work item: partial[item][0:ld] = sum over its rows x of
@@ -253,7 +255,19 @@ struct TcSoftmaxParams {
   int64_t zero_n4;
   int* status;
   int pdl;
+  // Early part of the step's decode (steady steps, U[o_t] formed by the
+  // gradient contraction): with pre_out set, the grid also writes
+  // pre_out[p] = B sum_{o != o_t} U[o][p] + sum_{deviating stores r}
+  // (b_r - B) sum_{o != o_t} store[r][o][p] for every float4 column p
+  // (pre: the step's decode arguments); the decode then adds the slot o_t
+  // terms (DecodeArgs::pre).
+  DecodeArgs pre;
+  float* pre_out = nullptr;
 };
+// Columns (float4) from which the step's decode is split this way, and the
+// deviating stores (CR: stragglers) it handles at most.
+constexpr int64_t kPreDecodeMinP4 = 1 << 18;
+constexpr int kPreMaxDev = 64;
 // Clusters of NT that fit at once (0: this NT is not supported).
 int tc_softmax_max_clusters(int NT);
 // tmXq: X, box {64, 128 / NT}; tmW: Wb, box {64, 128}; tmR: Rb, box {64, 32}

@@ -87,8 +87,12 @@ __device__ __forceinline__ int fr_rep(const DecodeArgs& a, int g) {
 }
 
 // One warp derives the plan; invalid masks set kErrBadMask.  It depends only
-// on the mask, so it can run before the step's gradients exist.
-__device__ __forceinline__ void derive_plan_warp(const DecodeArgs& a, DecodePlan& pl, int lane) {
+// on the mask, so it can run before the step's gradients exist.  Plan: a
+// DecodePlan, or a struct of the same members with shorter dev / devc arrays
+// (more deviating stores than they hold also set kErrBadMask).
+template <class Plan>
+__device__ __forceinline__ void derive_plan_warp(const DecodeArgs& a, Plan& pl, int lane) {
+  constexpr int kCap = (int)(sizeof(pl.dev) / sizeof(pl.dev[0]));
   const bool cr = a.scheme == PGC_CR;
   const float A = cr ? 1.0f / (float)((a.n - a.s) * a.c) : 1.0f / (float)a.n;
   int cnt = 0;
@@ -112,15 +116,17 @@ __device__ __forceinline__ void derive_plan_warp(const DecodeArgs& a, DecodePlan
     const unsigned bal = __ballot_sync(0xffffffffu, devr);
     if (devr) {
       const int pos = nd + __popc(bal & ((1u << lane) - 1u));
-      pl.dev[pos] = r;
-      pl.devc[pos] = br - A;
+      if (pos < kCap) {
+        pl.dev[pos] = r;
+        pl.devc[pos] = br - A;
+      }
     }
     nd += __popc(bal);
   }
   if (lane == 0) {
-    pl.ndev = nd;
+    pl.ndev = nd < kCap ? nd : kCap;
     pl.B = A;
-    if (cnt != a.s) atomicOr(a.status, kErrBadMask);
+    if (cnt != a.s || nd > kCap) atomicOr(a.status, kErrBadMask);
   }
   __syncwarp();
 }

@@ -39,7 +39,7 @@ constexpr int kFM = 128, kFN = 256, kFK = 64;
 constexpr int kFStages = 4;
 constexpr uint32_t kFA = kFM * kFK * 2;        // 16 KB A tile per stage
 constexpr uint32_t kFB = kFN * kFK * 2;        // 32 KB B tile per stage
-constexpr int kFThreads = 192;                 // producer, MMA, 4 epilogue warps
+constexpr int kFThreads = 320;                 // producer, MMA, 4 epilogue warps, 4 pre-decode warps
 constexpr uint32_t kFTmem = 2 * kFN;           // two fp32 accumulators
 constexpr uint32_t kRBox = 32 * 64 * 2;        // one 32-row x 64-class bf16 output box
 constexpr int kMaxNT = 8;
@@ -88,6 +88,14 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 struct FusedSmem {
   uint32_t sA, sB, box, stats, bars, total;
 };
+// The decode plan of the early decode terms, for at most kPreMaxDev stores
+// whose coefficient deviates (CR: the stragglers).
+struct PrePlan {
+  float B;
+  int ndev;
+  int dev[kPreMaxDev];
+  float devc[kPreMaxDev];
+};
 __host__ __device__ inline FusedSmem fused_smem(int NT) {
   FusedSmem s;
   s.sA = 0;
@@ -105,6 +113,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
 tc_logits_softmax_kernel(const __grid_constant__ CUtensorMap tmXq, const __grid_constant__ CUtensorMap tmW,
                          const __grid_constant__ CUtensorMap tmR, TcSoftmaxParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ PrePlan pre_plan;
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int NT = p.NT;
   const FusedSmem L = fused_smem(NT);
@@ -207,6 +216,48 @@ tc_logits_softmax_kernel(const __grid_constant__ CUtensorMap tmXq, const __grid_
       umma_commit(&acc_full[acc]);
     }
     if (!ok) atomicExch(cta_err, 1);
+  } else if (warp >= 6) {
+    // ---- pre-decode: the part of the step's decode that reads only data the
+    // step leaves as it is (§V-B decode with the slot-total form): for this
+    // CTA's slice of the float4 columns, pre = B sum_{o != o_t} U[o] +
+    // sum_{stores r with b_r != B} (b_r - B) sum_{o != o_t} store[r][o].  It
+    // streams beside the GEMM, so the decode after the gradient contraction
+    // reads only pre, U[o_t] and the deviating stores' slot o_t.
+    if (p.pre_out) {
+      const DecodeArgs& a = p.pre;
+      if (warp == 6) derive_plan_warp(a, pre_plan, lane);   // needs only the mask
+      asm volatile("bar.sync 1, 128;" ::: "memory");          // the four pre-decode warps
+      grid_dep_wait();                   // the stores and slot totals of the previous steps
+      const int64_t P4 = a.P / 4, slotP = (int64_t)a.c * P4;
+      const int c = a.c, sl = a.slot;
+      const int64_t q0 = P4 * blockIdx.x / gridDim.x, q1 = P4 * (blockIdx.x + 1) / gridDim.x;
+      const float4* U = reinterpret_cast<const float4*>(a.U);
+      const float4* store = reinterpret_cast<const float4*>(a.store);
+      for (int64_t pc = q0 + (threadIdx.x - 192); pc < q1; pc += 128) {
+        float4 V = f4zero(), D = f4zero();
+        for (int o0 = 0; o0 < c; o0 += 8) {
+          float4 v[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            v[j] = (o0 + j < c && o0 + j != sl) ? __ldcg(U + (int64_t)(o0 + j) * P4 + pc) : f4zero();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) V = f4add(V, v[j]);
+        }
+        for (int q = 0; q < pre_plan.ndev; ++q) {
+          const float4* base = store + (int64_t)pre_plan.dev[q] * slotP + pc;
+          float4 Cr = f4zero();
+          for (int o0 = 0; o0 < c; o0 += 8) {
+            float4 v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[j] = (o0 + j < c && o0 + j != sl) ? __ldcg(base + (int64_t)(o0 + j) * P4) : f4zero();
+#pragma unroll
+            for (int j = 0; j < 8; ++j) Cr = f4add(Cr, v[j]);
+          }
+          D = f4fma(pre_plan.devc[q], Cr, D);
+        }
+        reinterpret_cast<float4*>(p.pre_out)[pc] = f4fma(pre_plan.B, V, D);
+      }
+    }
   } else if (warp >= 2) {
     // ---- epilogue: softmax residual of this CTA's 256 classes ---------------
     const int q = warp & 3;
