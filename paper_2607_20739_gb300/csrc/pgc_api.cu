@@ -705,12 +705,23 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
     PGC_ALLOC(ctx->Z, std::max(zcc, ztc) * sizeof(float));
   }
   if (ctx->tc) PGC_ALLOC(ctx->Rb, (size_t)max_zpad * ctx->Ktc * sizeof(uint16_t));
-  // the early decode terms run in the fused logits kernel when the decode
-  // reads enough to pay for it (the one-thread-per-column decode sizes);
-  // PGC_NO_PRE_DECODE=1 leaves the whole decode after the contraction
-  if (ctx->tc && ctx->tcf && !gc_weighted && ctx->P / 4 >= kPreDecodeMinP4 && s <= kPreMaxDev &&
-      !(std::getenv("PGC_NO_PRE_DECODE") && std::getenv("PGC_NO_PRE_DECODE")[0] == '1'))
-    PGC_ALLOC(ctx->pre, Pb);
+  // The decode's terms of the slots other than o_t are summed by four warps
+  // of the fused logits kernel when that pays: the decode after the gradient
+  // contraction then reads (c - 1)(1 + s) P floats less (at about 6.5 TB/s),
+  // while the warps stream them at about 2.2 TB/s beside a GEMM running at
+  // about 1.43 PFLOP/s that gives up about 6 % to them and waits for them if
+  // it finishes first.  PGC_PRE_DECODE=1 (=0) forces the split on (off).
+  if (ctx->tc && ctx->tcf && !gc_weighted && ctx->P / 4 >= kPreDecodeMinP4 && s <= kPreMaxDev) {
+    const int cc = ctx->c;
+    const double rows_eval = scheme == PGC_CR ? (double)ctx->total_rows : (double)ctx->total_rows / cc;
+    const double pre_bytes = (double)(cc - 1) * (1 + (scheme == PGC_CR ? s : 0)) * (double)ctx->P * 4.0;
+    const double t_gemm = 2.0 * rows_eval * (double)ctx->ld * (double)ctx->Ktc / 1.43e15;
+    const double t_pre = pre_bytes / 2.2e12;
+    const double gain = pre_bytes / 6.5e12 - std::max(0.0, t_pre - t_gemm) - 0.06 * t_gemm;
+    bool on = gain > 0.0;
+    if (const char* e = std::getenv("PGC_PRE_DECODE")) on = e[0] == '1';
+    if (on) PGC_ALLOC(ctx->pre, Pb);
+  }
   PGC_ALLOC(ctx->coeff, (size_t)n * sizeof(float));
   PGC_ALLOC(ctx->status, sizeof(int));
   PGC_ALLOC(ctx->loss_blocks, (size_t)ctx->loss_nblocks * sizeof(double));

@@ -105,6 +105,22 @@ def test_parity_gradient_runs(libpgc, cuda, monkeypatch, run):
     g.close()
 
 
+@pytest.mark.parametrize("name", ["cr_tc_wide_decode", "fr_tc_wide_decode"])
+def test_parity_early_decode_terms(libpgc, cuda, monkeypatch, name):
+    """The decode split around the tensor-core GEMMs, forced on for cases too
+    small for it to pay (the full-size cr_n128_softmax_k1000 runs take it by
+    default): the logits kernel sums the terms of the slots other than o_t,
+    the decode after the contraction adds the slot o_t terms."""
+    monkeypatch.setenv("PGC_PRE_DECODE", "1")
+    w, T = CASES[name]
+    Xs, ys, masks = generate(w, T)
+    g, grecs = run_gpu(libpgc, w, Xs, ys, masks)
+    assert g.gradient_path == "tc_fused"
+    orecs = run_oracle(w, Xs, ys, masks)
+    compare_runs(w, grecs, orecs)
+    g.close()
+
+
 def test_parity_unfused_tensor_core_path(libpgc, cuda, monkeypatch):
     """A class count the fused kernel covers, forced through the three-kernel
     fall-back (logits GEMM, residual kernel, gradient contraction)."""
