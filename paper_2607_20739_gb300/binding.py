@@ -50,7 +50,7 @@ _sig = {
     "pgc_create_mode": (C.c_int, [C.POINTER(_vp), _i32, _i32, _i32, _i32, _i32, _i32, _i64, _i64, C.POINTER(_i64), C.c_float,
                              C.POINTER(C.c_float), _vp]),
     "pgc_load_partitions": (C.c_int, [_vp, C.POINTER(_vp), C.POINTER(_vp), _i32]),
-    "pgc_step": (C.c_int, [_vp, C.POINTER(C.c_uint8), _vp, _vp, _i32, C.POINTER(StepInfo)]),
+    "pgc_step": (C.c_int, [_vp, _vp, _vp, _vp, _i32, C.POINTER(StepInfo)]),
     "pgc_loss": (C.c_int, [_vp, C.POINTER(C.c_double)]),
     "pgc_sync": (C.c_int, [_vp]),
     "pgc_destroy": (C.c_int, [_vp]),
@@ -214,7 +214,9 @@ class PGC:
     def step(self, mask, grad_out=None, w_out=None, info: bool = True):
         """One training step.  Outputs may be numpy (host, waits) or torch CUDA
         tensors (device, returns immediately)."""
-        m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8))
+        m = mask
+        if not (type(m) is np.ndarray and m.dtype == np.uint8 and m.flags.c_contiguous):
+            m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8))
         if m.shape != (self.n,):
             raise ValueError("mask must have n entries")
         on_dev = 0
@@ -226,7 +228,7 @@ class PGC:
             gi = StepInfo()
             gi.eval_partition = self._eval.ctypes.data_as(C.POINTER(_i32))
             gi.fr_rep = self._rep.ctypes.data_as(C.POINTER(_i32))
-        _check(lib.pgc_step(self._h, m.ctypes.data_as(C.POINTER(C.c_uint8)),
+        _check(lib.pgc_step(self._h, m.ctypes.data,
                             _ptr(grad_out) if grad_out is not None else None,
                             _ptr(w_out) if w_out is not None else None, on_dev,
                             C.byref(gi) if gi is not None else None), "pgc_step")

@@ -140,6 +140,7 @@ struct pgc_ctx {
   int64_t Ktc = 0;           // classes padded to the forward N tile (256)
   uint16_t* Rb = nullptr;    // bf16 residuals [zpad rows][Ktc]
   float* pre = nullptr;      // fused tensor-core path: the decode's early terms [P]
+  int* status_h = nullptr;   // pinned host copy of the status word
   alignas(64) unsigned char tmXk[128];   // X as K-major A   (box 64 x 128)
   alignas(64) unsigned char tmW[128];    // Wb as K-major B  (box 64 x 128: one CTA's half of a 256 tile)
   alignas(64) unsigned char tmR[128];    // R as MN-major A  (box 64 x 64)
@@ -195,10 +196,11 @@ int cuda_fail(pgc_ctx* ctx, cudaError_t e) {
 
 // Read and clear nothing: map the device status word to a code.
 int read_status(pgc_ctx* ctx) {
-  int h = 0;
-  cudaError_t e = cudaMemcpyAsync(&h, ctx->status, sizeof(int), cudaMemcpyDeviceToHost, ctx->stream);
+  // into pinned memory: the copy is a plain asynchronous one, no staging
+  cudaError_t e = cudaMemcpyAsync(ctx->status_h, ctx->status, sizeof(int), cudaMemcpyDeviceToHost, ctx->stream);
   if (e == cudaSuccess) e = cudaStreamSynchronize(ctx->stream);
   if (e != cudaSuccess) return cuda_fail(ctx, e);
+  const int h = *ctx->status_h;
   if (h & kErrWaitTimeout) { ctx->broken = true; return PGC_ETIMEOUT; }
   if (h & kErrBadMask) { ctx->broken = true; return PGC_EMASK; }
   if (h & kErrSingular) { ctx->broken = true; return PGC_ESINGULAR; }
@@ -434,6 +436,8 @@ void free_all(pgc_ctx* ctx) {
                   ctx->gc_coeff, ctx->gc_d, ctx->gc_draws, ctx->gc_wts, ctx->pre};
   for (void* p : ptrs)
     if (p) cudaFree(p);
+  if (ctx->status_h) cudaFreeHost(ctx->status_h);
+  ctx->status_h = nullptr;
 }
 
 // Device address of a pinned host buffer mapped into the current device's
@@ -724,6 +728,10 @@ int pgc_create_mode(pgc_ctx** out, int32_t mode, int32_t n, int32_t s, int32_t s
   }
   PGC_ALLOC(ctx->coeff, (size_t)n * sizeof(float));
   PGC_ALLOC(ctx->status, sizeof(int));
+  {
+    cudaError_t _e = cudaMallocHost((void**)&ctx->status_h, sizeof(int));
+    if (_e != cudaSuccess) return fail(_e);
+  }
   PGC_ALLOC(ctx->loss_blocks, (size_t)ctx->loss_nblocks * sizeof(double));
   PGC_ALLOC(ctx->loss_out, sizeof(double));
   PGC_ALLOC(ctx->tables, tab.size());
